@@ -1,0 +1,133 @@
+"""Model shapes and workloads of the five synthetic decoder configurations.
+
+These are workload descriptions only (shapes, seeds, lengths); no arithmetic of
+the forward pass lives here.  The paper evaluates llama.cpp inference on
+Qwen3/Falcon GGUF models (Sec. 5.1, Tab. 1) without giving their internals, so
+the shapes are the standard Llama-3 / Qwen2.5 ones with seeded random bf16
+weights ~N(0, 0.02) and all RMSNorm gains equal to 1.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field, replace
+
+
+@dataclass(frozen=True)
+class ModelConfig:
+    name: str
+    n_layers: int
+    hidden: int
+    n_q_heads: int
+    n_kv_heads: int
+    head_dim: int
+    ffn_dim: int
+    vocab: int
+    rope_theta: float
+    rms_eps: float = 1e-5
+    tied_embeddings: bool = False
+    qkv_bias: bool = False
+    weight_std: float = 0.02
+    weight_seed: int = 0
+    # workload: `turns` rounds of (prompt_len-token chunk, then decode_steps greedy tokens)
+    prompt_len: int = 32
+    decode_steps: int = 16
+    turns: int = 1
+    prompt_seeds: tuple = (1,)
+    max_chunk: int = 2048
+    page_tokens: int = 16
+    extra: dict = field(default_factory=dict, compare=False)
+
+    @property
+    def q_dim(self) -> int:
+        return self.n_q_heads * self.head_dim
+
+    @property
+    def kv_dim(self) -> int:
+        return self.n_kv_heads * self.head_dim
+
+    @property
+    def total_tokens(self) -> int:
+        return self.turns * (self.prompt_len + self.decode_steps)
+
+    def with_(self, **kw) -> "ModelConfig":
+        return replace(self, **kw)
+
+
+TINY = ModelConfig(
+    name="tiny", n_layers=2, hidden=256, n_q_heads=4, n_kv_heads=2, head_dim=64,
+    ffn_dim=688, vocab=1024, rope_theta=10000.0, rms_eps=1e-5,
+    prompt_len=32, decode_steps=16)
+
+LLAMA_1B = ModelConfig(
+    name="llama3.2-1b", n_layers=16, hidden=2048, n_q_heads=32, n_kv_heads=8, head_dim=64,
+    ffn_dim=8192, vocab=128256, rope_theta=500000.0, rms_eps=1e-5, tied_embeddings=True,
+    prompt_len=512, decode_steps=128)
+
+LLAMA_8B = ModelConfig(
+    name="llama3-8b", n_layers=32, hidden=4096, n_q_heads=32, n_kv_heads=8, head_dim=128,
+    ffn_dim=14336, vocab=128256, rope_theta=500000.0, rms_eps=1e-5,
+    prompt_len=1024, decode_steps=256)
+
+LLAMA_8B_AGENTIC = LLAMA_8B.with_(
+    name="llama3-8b-agentic", prompt_len=2048, decode_steps=64, turns=4,
+    prompt_seeds=(1, 2, 3, 4))
+
+QWEN_14B = ModelConfig(
+    name="qwen2.5-14b", n_layers=48, hidden=5120, n_q_heads=40, n_kv_heads=8, head_dim=128,
+    ffn_dim=13824, vocab=152064, rope_theta=1000000.0, rms_eps=1e-6, qkv_bias=True,
+    prompt_len=2048, decode_steps=256)
+
+CONFIGS = {c.name: c for c in (TINY, LLAMA_1B, LLAMA_8B, LLAMA_8B_AGENTIC, QWEN_14B)}
+
+
+def tensor_specs(cfg: ModelConfig):
+    """Canonical tensor list: (name, (rows, cols), kind) with kind 'normal' or 'ones'.
+
+    The position of a tensor in this list is its generator tag.  All matrices
+    are row-major [out, in]; y = W x.
+    """
+    H, d = cfg.hidden, cfg.head_dim
+    specs = [("embed", (cfg.vocab, H), "normal")]
+    for l in range(cfg.n_layers):
+        p = f"layers.{l}."
+        specs.append((p + "attn_norm", (1, H), "ones"))
+        specs.append((p + "wq", (cfg.n_q_heads * d, H), "normal"))
+        specs.append((p + "wk", (cfg.n_kv_heads * d, H), "normal"))
+        specs.append((p + "wv", (cfg.n_kv_heads * d, H), "normal"))
+        if cfg.qkv_bias:
+            specs.append((p + "bq", (1, cfg.n_q_heads * d), "normal"))
+            specs.append((p + "bk", (1, cfg.n_kv_heads * d), "normal"))
+            specs.append((p + "bv", (1, cfg.n_kv_heads * d), "normal"))
+        specs.append((p + "wo", (H, cfg.n_q_heads * d), "normal"))
+        specs.append((p + "ffn_norm", (1, H), "ones"))
+        specs.append((p + "wg", (cfg.ffn_dim, H), "normal"))
+        specs.append((p + "wu", (cfg.ffn_dim, H), "normal"))
+        specs.append((p + "wd", (H, cfg.ffn_dim), "normal"))
+    specs.append(("final_norm", (1, H), "ones"))
+    if not cfg.tied_embeddings:
+        specs.append(("lm_head", (cfg.vocab, H), "normal"))
+    return specs
+
+
+def decode_bytes_per_token(cfg: ModelConfig, ctx: int) -> int:
+    """Algorithmic HBM bytes one decode step must read: every weight once plus
+    the K and V of `ctx` cached positions (bf16)."""
+    n = 0
+    for name, (r, c), _ in tensor_specs(cfg):
+        if name == "embed":
+            n += cfg.hidden            # one embedding row is gathered
+        else:
+            n += r * c
+    if cfg.tied_embeddings:
+        n += cfg.vocab * cfg.hidden    # the LM head reads the (shared) embedding table
+    return 2 * n + cfg.n_layers * 2 * cfg.kv_dim * 2 * ctx
+
+
+def prefill_flops(cfg: ModelConfig, T: int, P: int = 0) -> float:
+    """Algorithmic FLOPs of a T-token prefill appended after P cached tokens:
+    2*T*(per-layer linear params)*L + causal attention (unmasked pairs only,
+    QK^T and PV) + the LM head on the last row."""
+    H, d = cfg.hidden, cfg.head_dim
+    lin = H * (cfg.q_dim + 2 * cfg.kv_dim) + cfg.q_dim * H + 3 * H * cfg.ffn_dim
+    pairs = T * P + T * (T + 1) // 2
+    attn = cfg.n_q_heads * d * 4 * pairs
+    return float(2 * T * lin * cfg.n_layers + attn * cfg.n_layers + 2 * cfg.vocab * H)
