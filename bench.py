@@ -1,0 +1,314 @@
+"""Benchmark of the batch-1 decoder forward pass on the Llama-3-8B shape.
+
+One step = one request: reset, prefill of a 1024-token seeded prompt (TTFT),
+then 256 greedy decode steps, all through the C ABI of libwici.so.  `value` is
+decode tokens/s over the K timed steps (CUDA events on the library's stream;
+weights and KV already in HBM); TTFT and achieved HBM bandwidth are reported
+beside it.  The 16 GB of weights exceed L2 (129 MB) many times over, so no L2
+flush is needed between steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the CPU oracle (numpy fp64) on a bounded sample of the
+same workload: it is the baseline this path is compared with.  With N > 1 the
+job runs as N independent replicas (one per GPU, launched by torchrun): the
+decode path has no exchange step, so there is no collective.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import gen  # noqa: E402
+
+CFG = gen.LLAMA_8B
+PROMPT = CFG.prompt_len        # 1024
+DECODE = CFG.decode_steps      # 256
+METRIC = "bs=1 decode tok/s (Llama-3-8B shape, 1024-token prompt, 256 greedy steps)"
+NOMINAL_HBM_GBS = 8000.0
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"]),
+                "bf16_tflops_sustained": float(d.get("bf16_tflops_sustained", d["bf16_tflops"])),
+                "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples every 200 ms while running."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [s for s in sm if s > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(smax), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def cpu_oracle_sample(weights, budget_s: float = 20.0):
+    """The oracle as it stands on the host cores: a 16-token prompt, then greedy
+    decode steps until about `budget_s` of decode time (at least 1)."""
+    import oracle
+    m = oracle.OracleModel(CFG, weights, max_tokens=64)
+    _, tok = m.prefill(gen.make_prompt(CFG, 16, seed=1))
+    n, t0 = 0, time.perf_counter()
+    while True:
+        _, tok = m.decode(tok)
+        n += 1
+        if time.perf_counter() - t0 > budget_s or n >= 8:
+            break
+    dt = time.perf_counter() - t0
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return {"value": n / dt, "unit": "tok/s", "cores": cores, "kind": "oracle",
+            "sample": f"{CFG.name} weights, 16-token prompt, {n} greedy decode steps at context 17..{16 + n} "
+                      f"(numpy fp64, {dt:.1f} s)"}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    t0 = time.time()
+    weights = gen.make_weights(CFG)
+    budget = max(5.0, 20.0 * args.steps / max(args.steps, 1))
+    samples = []
+    for _ in range(args.warmup + args.steps):
+        samples.append(cpu_oracle_sample(weights, budget_s=budget / max(1, args.steps)))
+    timed = samples[args.warmup:]
+    val = statistics.median(s["value"] for s in timed)
+    cb = dict(timed[-1])
+    cb["value"] = val
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "tok/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 / val,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded bf16 weights ~N(0,0.02), uniform-random prompt tokens)",
+            "config": {"workload": f"{CFG.name}: prompt {PROMPT}, {DECODE} greedy decode steps (oracle sample)"},
+            "cpu_baseline": cb,
+            "e2e": {"value": val, "unit": "tok/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "wall_s": time.time() - t0}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours(args):
+    import torch
+    from paper_2608_24204_gb300 import WiciModel, wici
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.cuda.current_device()
+    pk = peaks()
+
+    t_setup = time.time()
+    weights = gen.make_weights(CFG)
+    max_tokens = PROMPT + DECODE + 16
+    model = WiciModel(CFG, max_tokens=max_tokens, max_chunk=PROMPT).load(weights)
+    prompt = gen.make_prompt(CFG, PROMPT, seed=1)
+    stream = model.stream
+
+    def one_request(ev=None):
+        model.reset()
+        if ev:
+            ev[0].record(stream)
+        model.prefill(prompt)
+        if ev:
+            ev[1].record(stream)
+        model.decode(DECODE)
+        if ev:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        one_request()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    clocks = ClockSampler(dev)
+    clocks.start()
+    barrier()
+    g0 = torch.cuda.Event(enable_timing=True)
+    g1 = torch.cuda.Event(enable_timing=True)
+    g0.record(stream)
+    for k in range(args.steps):
+        one_request(evs[k])
+    g1.record(stream)
+    barrier()
+    clk = clocks.stop()
+    total_ms = g0.elapsed_time(g1)
+    ttft = [e[0].elapsed_time(e[1]) for e in evs]
+    dec = [e[1].elapsed_time(e[2]) for e in evs]
+    dec_s = sum(dec) / 1000.0
+    local_tok = args.steps * DECODE
+    t_max = torch.tensor([dec_s, total_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        torch.distributed.all_reduce(t_max, op=torch.distributed.ReduceOp.MAX)
+    dec_s_max, total_ms_max = float(t_max[0]), float(t_max[1])
+    value = world * local_tok / dec_s_max
+
+    # bytes per decoded token (weights + KV of the context), averaged over the 256 steps
+    bytes_tok = sum(gen.decode_bytes_per_token(CFG, PROMPT + i) for i in range(1, DECODE + 1)) / DECODE
+    step_gbs = bytes_tok * (local_tok / dec_s) / 1e9
+
+    # roofline of the dominant kernel (gate/up + SwiGLU GEMV), timed live with CUDA events
+    model.reset()
+    model.prefill(prompt)
+    prof = wici.wici_profile_decode(model.ctx, 8)
+    H, F = CFG.hidden, CFG.ffn_dim
+    gu_bytes = 2 * F * H * 2 + H * 2 + H * 4 + F * 4   # Wg|Wu + gain + x read + m written
+    n_gu, ms_gu = prof["gate_up_swiglu"]
+    gu_gbs = gu_bytes / (ms_gu / n_gu / 1000.0) / 1e9
+    roofline = {"bound": "hbm", "kernel": "gate_up_swiglu", "achieved": gu_gbs, "peak": pk["hbm_gbs"],
+                "unit": "GB/s", "frac": gu_gbs / pk["hbm_gbs"], "traffic": None,
+                "peak_source": pk["source"], "bytes_per_launch": gu_bytes,
+                "avg_launch_us": ms_gu / n_gu * 1000.0}
+    kernel_share = {k: {"launches": v[0], "ms": v[1]} for k, v in prof.items()}
+
+    # end to end through the public API: host prompt in pinned memory, one C-ABI call per token
+    pinned = torch.from_numpy(prompt.copy()).pin_memory()
+    host_prompt = pinned.numpy()
+    e2e_steps = max(1, min(2, args.steps))
+    e2e_dec, e2e_ttft = [], []
+    for _ in range(e2e_steps):
+        model.reset()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        tok = model.prefill(host_prompt)
+        t1 = time.perf_counter()
+        for _ in range(DECODE):
+            tok = model.decode_step(-1)
+        t2 = time.perf_counter()
+        e2e_ttft.append((t1 - t0) * 1000)
+        e2e_dec.append(t2 - t1)
+    e2e_val = world * DECODE * e2e_steps / sum(e2e_dec)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_oracle_sample(weights, budget_s=15.0)
+
+    launches_per_step = (1 + CFG.n_layers * 7 + 1) + DECODE * (5 * CFG.n_layers + 1)
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tok/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms_max / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded bf16 weights ~N(0,0.02), uniform-random prompt tokens)",
+            "config": {"workload": f"{CFG.name}: L=32 H=4096 32q/8kv d=128 F=14336 V=128256; prompt {PROMPT}, "
+                                   f"{DECODE} greedy decode steps per request",
+                       "l2": "inputs larger than L2 (16 GB of weights streamed per token)",
+                       "parallelism": "replicas" if world > 1 else "single GPU",
+                       "accumulate": "fp32"},
+            "ttft_ms": statistics.median(ttft),
+            "decode_ms_per_token": dec_s / local_tok * 1000.0,
+            "decode_gbs": step_gbs, "decode_frac_of_8tbs": step_gbs / (NOMINAL_HBM_GBS),
+            "decode_frac_of_measured_hbm": step_gbs / pk["hbm_gbs"],
+            "bytes_per_token": bytes_tok,
+            "prefill_tflops": gen.prefill_flops(CFG, PROMPT) / (statistics.median(ttft) / 1000.0) / 1e12,
+            "roofline": roofline, "kernels": kernel_share, "cpu_baseline": cpu,
+            "e2e": {"value": e2e_val, "unit": "tok/s", "h2d_bytes_per_step": PROMPT * 4,
+                    "d2h_bytes_per_step": (DECODE + 1) * 4, "ttft_ms": statistics.median(e2e_ttft),
+                    "how": "wici_prefill from pinned host tokens, then one wici_decode_step call per token, "
+                           "wall clock"},
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clk,
+            "setup_s": time.time() - t_setup,
+        }
+        print(json.dumps(line), flush=True)
+    model.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

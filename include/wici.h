@@ -1,0 +1,158 @@
+/*
+ * wici.h - C ABI of the GB300-native batch-1 decoder forward pass.
+ *
+ * The library computes the per-token GPU work that WiCi (arxiv 2608.24204)
+ * offloads from a mobile client: T_Local of Eq. 1 (Sec. 3.3), i.e. the
+ * prefill over a prompt (time to first token) and then one forward step per
+ * generated token, each step repeating the same computation with a new input
+ * token (Sec. 4.2.2).  Model: Llama-style decoder (RMSNorm, rotate-half RoPE,
+ * grouped-query causal attention over a paged bf16 KV cache, SwiGLU MLP,
+ * greedy argmax); weights are bf16, row-major [out, in], y = W x.
+ *
+ * Conventions for every entry point
+ *   - Return value: WICI_OK (0) or a negative wici_status; the message is in
+ *     wici_last_error(ctx) (ctx may be NULL for wici_create/wici_get_sizes
+ *     failures: the message is then per calling thread).
+ *   - On any error the KV length and the cached K/V of positions < kv_len are
+ *     unchanged.  Capacity and arguments are checked before any launch.
+ *   - Device buffers (weights arena, KV pool, workspace) are allocated by the
+ *     caller with the sizes from wici_get_sizes and borrowed by the context
+ *     until wici_destroy; the library owns only its streams, events, CUDA
+ *     graph and a small pinned staging buffer.
+ *   - Host buffers (token arrays, logits) are owned by the caller and are
+ *     read or written before the call returns: every call that produces
+ *     output synchronises its stream before returning.
+ *   - A context is not thread-safe; use one per thread (the paper's router
+ *     serves each client from its own thread, Sec. 3.2).
+ *   - Device-side waits are bounded in time; a wait that gives up makes the
+ *     call return WICI_E_TIMEOUT and leaves the context usable.
+ */
+#ifndef WICI_H
+#define WICI_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct wici_ctx wici_ctx;
+
+typedef enum wici_status {
+    WICI_OK = 0,
+    WICI_E_ARG = -1,      /* bad pointer, size, name or configuration */
+    WICI_E_STATE = -2,    /* call not valid now (e.g. decode before prefill, weights missing) */
+    WICI_E_CAPACITY = -3, /* the tokens would not fit in max_tokens KV positions */
+    WICI_E_CUDA = -4,     /* a CUDA runtime call failed */
+    WICI_E_TIMEOUT = -5   /* a bounded device-side wait gave up */
+} wici_status;
+
+/* Model shape and capacity.  Constraints: hidden, ffn_dim and n_q_heads*head_dim
+ * multiples of 8; head_dim 64 or 128; n_q_heads a multiple of n_kv_heads with at
+ * most 8 query heads per KV head; page_tokens == 16; 1 <= max_chunk <= max_tokens. */
+typedef struct wici_config {
+    int32_t n_layers, hidden, n_q_heads, n_kv_heads, head_dim, ffn_dim, vocab;
+    int32_t max_tokens;      /* KV capacity in positions */
+    int32_t max_chunk;       /* tokens processed per prefill pass; longer prompts are split */
+    int32_t page_tokens;     /* KV page size in tokens (16) */
+    float rms_eps;
+    double rope_theta;
+    int32_t tied_embeddings; /* 1: the LM head is the embedding table */
+    int32_t qkv_bias;        /* 1: bq, bk, bv are present (added before RoPE) */
+} wici_config;
+
+/* Device bytes the caller allocates (each buffer 256-byte aligned). */
+typedef struct wici_sizes {
+    size_t weight_bytes;     /* packed bf16 weight arena */
+    size_t kv_bytes;         /* paged bf16 K/V pool: [layer][page][K|V][kv_head][16][head_dim] */
+    size_t workspace_bytes;  /* activations, partials, RoPE table, page table, control words */
+} wici_sizes;
+
+/* One named weight tensor, bf16 row-major [rows, cols].  Names:
+ *   "embed" [vocab, hidden]; "final_norm" [1, hidden]; "lm_head" [vocab, hidden] (untied);
+ *   "layers.<l>.attn_norm" [1, hidden]; "layers.<l>.wq" [n_q*d, hidden];
+ *   "layers.<l>.wk" / ".wv" [n_kv*d, hidden]; "layers.<l>.bq" [1, n_q*d] and
+ *   ".bk" / ".bv" [1, n_kv*d] (qkv_bias only); "layers.<l>.wo" [hidden, n_q*d];
+ *   "layers.<l>.ffn_norm" [1, hidden]; "layers.<l>.wg" / ".wu" [ffn, hidden];
+ *   "layers.<l>.wd" [hidden, ffn].
+ * `data` is a host pointer (on_device = 0) or a device pointer (on_device = 1);
+ * it is read during the call and not kept.  The paper's frameworks load a model
+ * "tensor by tensor" (Sec. 4.1); so does this call. */
+typedef struct wici_tensor {
+    const char *name;
+    const void *data;
+    int64_t rows, cols;
+    int32_t on_device;
+} wici_tensor;
+
+/* Sizes of the three caller-owned device buffers for `cfg`.  WICI_E_ARG on an
+ * invalid configuration. */
+int wici_get_sizes(const wici_config *cfg, wici_sizes *out);
+
+/* Create a context on the current CUDA device.  `cuda_stream` (a cudaStream_t,
+ * may be NULL for the legacy stream) orders every launch of this context; the
+ * three buffers must be at least wici_get_sizes() bytes and 256-byte aligned.
+ * The KV page table starts as the identity.  *out receives the context. */
+int wici_create(const wici_config *cfg, void *cuda_stream, void *weight_dev, void *kv_dev,
+                void *workspace_dev, wici_ctx **out);
+
+/* Copy `n` named tensors into the packed weight arena (rows of Wq/Wk are paired
+ * for RoPE, Wg/Wu rows are interleaved, Wq/Wk/Wv are concatenated).  May be
+ * called several times; prefill/decode require every tensor to have been loaded. */
+int wici_load_weights(wici_ctx *ctx, const wici_tensor *t, int32_t n);
+
+/* Append `n` >= 1 host tokens at positions kv_len..kv_len+n-1 (Sec. 5.1 TTFT
+ * path; a later call after decode steps is a chunked prefill onto the live cache).
+ * logits_out (nullable, host float[vocab]) receives the last position's logits;
+ * token_out (nullable) its greedy token.  WICI_E_CAPACITY if kv_len+n > max_tokens,
+ * WICI_E_ARG if a token is outside [0, vocab). */
+int wici_prefill(wici_ctx *ctx, const int32_t *tokens, int32_t n, float *logits_out,
+                 int32_t *token_out);
+
+/* One decode step: feed `token_in` (>= 0), or the last greedy token when
+ * token_in < 0, at position kv_len; kv_len += 1.  Outputs as for wici_prefill.
+ * Runs the captured CUDA graph of the whole step.  WICI_E_STATE before the
+ * first prefill. */
+int wici_decode_step(wici_ctx *ctx, int32_t token_in, float *logits_out, int32_t *token_out);
+
+/* `n_steps` greedy decode steps back to back on the device (each step feeds
+ * the previous step's argmax; the first feeds token_in, or the last greedy
+ * token if token_in < 0).  tokens_out (nullable, host int32[n_steps]) receives
+ * the generated tokens. */
+int wici_decode(wici_ctx *ctx, int32_t n_steps, int32_t token_in, int32_t *tokens_out);
+
+/* Forget the cached tokens (kv_len := 0); weights stay loaded. */
+int wici_reset(wici_ctx *ctx);
+
+/* Replace the logical->physical KV page map (host int32[n], n = max_tokens/16
+ * rounded up, a permutation of 0..n-1).  Only valid when kv_len == 0. */
+int wici_set_page_table(wici_ctx *ctx, const int32_t *pages, int32_t n);
+
+/* Number of cached positions, or a negative status. */
+int32_t wici_kv_len(const wici_ctx *ctx);
+
+/* Message of the last error on ctx (or of this thread when ctx is NULL). */
+const char *wici_last_error(const wici_ctx *ctx);
+
+/* Per-kernel timing of `n_steps` decode steps run as individual launches, each
+ * bracketed by CUDA events on the context's stream (for roofline accounting).
+ * For each kernel kind i < *n_kinds: names[i] (static string), launches[i] and
+ * total_ms[i].  Arrays have room for `cap` entries.  Advances kv_len by n_steps
+ * like wici_decode. */
+int wici_profile_decode(wici_ctx *ctx, int32_t n_steps, const char **names, int32_t *launches,
+                        double *total_ms, int32_t cap, int32_t *n_kinds);
+
+/* Self-test of the bounded device wait: launches one CTA that waits on an
+ * mbarrier nobody arrives at, giving up after `limit_ns` nanoseconds.  Returns
+ * WICI_E_TIMEOUT when the wait gave up as designed (the expected result). */
+int wici_check_bounded_wait(void *cuda_stream, int64_t limit_ns);
+
+/* Destroy the context (frees only what the library allocated). */
+void wici_destroy(wici_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WICI_H */

@@ -1,0 +1,66 @@
+// Device buffers and the enqueue functions of the decode and prefill paths.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "plan.h"
+
+namespace wici {
+
+// Device pointers derived from the three caller-owned buffers and the plan.
+struct Bufs {
+    uint16_t *W;      // packed weight arena (bf16 bits)
+    uint16_t *KV;     // paged KV pool (bf16 bits)
+    int *ctrl;        // control words (CtrlSlot)
+    int *hist;        // hist[p] = greedy token produced for position p   [max_tokens + 1]
+    float *x;         // decode residual stream                             [H]
+    float *q;         // decode query after RoPE                            [qdim]
+    float *o;         // decode attention output                            [qdim]
+    float *m;         // decode SwiGLU output                               [F]
+    float *logits;    // last logits                                        [V]
+    int2 *amax;       // per-CTA argmax partials (value bits, index)        [num_sms]
+    float *attn;      // flash-decode partials [nkv][splits][group][d + 2]
+    float2 *rope;     // (cos, sin) of p * theta^(-2i/d)                     [max_tokens][d/2]
+    int *pages;       // logical -> physical KV page                         [max_pages]
+    int *tok;         // prefill chunk tokens                                [max_chunk]
+    float *X;         // prefill residual stream                             [max_chunk][H]
+    float *A;         // prefill GEMM input rows (fp32)                      [max_chunk][max(H,F,qdim)]
+    float *Q;         // prefill queries after RoPE                          [max_chunk][qdim]
+    float *O;         // prefill attention output                            [max_chunk][qdim]
+    float *M;         // prefill SwiGLU output                               [max_chunk][F]
+};
+
+// Called around every launch when profiling (eager mode).
+struct LaunchHook {
+    virtual void before(const char *name) = 0;
+    virtual void after(const char *name) = 0;
+    virtual ~LaunchHook() {}
+};
+
+// One-time per-process kernel attributes (dynamic shared memory limits).
+cudaError_t setup_kernels();
+
+// Whole decode step for the token in ctrl[CTRL_TOKEN] at position ctrl[CTRL_POS]:
+// 5 launches per layer + the LM head.  `pdl` enables programmatic dependent launch.
+cudaError_t enqueue_decode_step(const Plan &p, const Bufs &b, cudaStream_t st, bool pdl,
+                                LaunchHook *hook);
+
+// Final RMSNorm + LM head + argmax of the row in b.x; the last CTA writes
+// ctrl[CTRL_TOKEN], hist[pos + pos_add] and advances ctrl[CTRL_POS] by pos_add.
+cudaError_t enqueue_lm_head(const Plan &p, const Bufs &b, cudaStream_t st, bool pdl, int pos_add,
+                            LaunchHook *hook);
+
+// Prefill of the chunk b.tok[0..T) at positions P..P+T-1 through every layer.
+// With lm_pos_add > 0 it then copies the chunk's last row to b.x and runs the
+// LM head, which advances ctrl[CTRL_POS] by lm_pos_add.
+cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, cudaStream_t st, int P, int T,
+                                  int lm_pos_add, LaunchHook *hook);
+
+// RoPE table for positions [0, max_tokens).
+cudaError_t enqueue_rope_table(const Plan &p, const Bufs &b, cudaStream_t st);
+
+// One CTA waiting on an mbarrier that never completes; writes the wait's
+// site id to *err when it gives up after limit_ns.
+cudaError_t enqueue_bounded_wait_probe(int *err, int64_t limit_ns, cudaStream_t st);
+
+}  // namespace wici

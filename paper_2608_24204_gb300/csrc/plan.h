@@ -1,0 +1,45 @@
+// Buffer plan: where every tensor lives in the caller-owned weight arena,
+// KV pool and workspace.  Host-side only; shared by the launch code.
+#pragma once
+#include <stddef.h>
+#include <stdint.h>
+
+#include <vector>
+
+#include "../../include/wici.h"
+
+namespace wici {
+
+constexpr int kPage = 16;          // tokens per KV page
+constexpr int kGemvThreads = 288;  // 8 consumer warps + 1 producer warp
+constexpr int kGemvStages = 3;     // ring depth
+constexpr uint32_t kGemvStageMax = 32768;  // bytes per stage (one row of K <= 16384)
+constexpr int kGemvMaxRows = 64;   // rows per stage (bounded by the reduction scratch)
+
+struct LayerOffsets {       // bf16 element offsets into the weight arena
+    size_t attn_norm, wqkv, bqkv, wo, ffn_norm, wgu, wd;
+};
+
+struct Plan {
+    wici_config cfg;
+    int L, H, F, V, nq, nkv, d, qdim, kvdim, nqkv, group, max_pages, max_chunk;
+    // weight arena (bf16 elements)
+    size_t w_embed, w_final_norm, w_lm;
+    std::vector<LayerOffsets> layer;
+    size_t weight_elems;
+    // KV pool (bf16 elements)
+    size_t kv_page_elems;   // one page: [K|V][nkv][16][d]
+    size_t kv_layer_elems;  // max_pages pages
+    size_t kv_elems;
+    // workspace (byte offsets)
+    size_t ws_ctrl, ws_hist, ws_x, ws_q, ws_o, ws_m, ws_logits, ws_amax, ws_attn, ws_rope,
+        ws_pages, ws_tok, ws_X, ws_A, ws_Q, ws_O, ws_M;
+    size_t ws_bytes;
+    int attn_splits;        // flash-decode splits per KV head
+    int num_sms;
+};
+
+// Fills `p` from `cfg`; returns an error message or nullptr.
+const char *make_plan(const wici_config *cfg, int num_sms, Plan *p);
+
+}  // namespace wici
