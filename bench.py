@@ -35,6 +35,7 @@ import gen  # noqa: E402
 CFG = gen.LLAMA_8B
 PROMPT = CFG.prompt_len        # 1024
 DECODE = CFG.decode_steps      # 256
+QUICK = False                  # profiling runs: no e2e, no per-kernel pass, no CPU baseline
 METRIC = "bs=1 decode tok/s (Llama-3-8B shape, 1024-token prompt, 256 greedy steps)"
 NOMINAL_HBM_GBS = 8000.0
 
@@ -158,6 +159,12 @@ def run_reference(args):
 
 
 def run_ours(args):
+    global CFG, DECODE, QUICK
+    if args.layers:
+        CFG = CFG.with_(name=f"{CFG.name}-{args.layers}l", n_layers=args.layers)
+    if args.decode_steps:
+        DECODE = args.decode_steps
+    QUICK = args.quick
     import torch
     from paper_2608_24204_gb300 import WiciModel, wici
 
@@ -224,6 +231,13 @@ def run_ours(args):
     # bytes per decoded token (weights + KV of the context), averaged over the 256 steps
     bytes_tok = sum(gen.decode_bytes_per_token(CFG, PROMPT + i) for i in range(1, DECODE + 1)) / DECODE
     step_gbs = bytes_tok * (local_tok / dec_s) / 1e9
+
+    if QUICK:
+        if rank == 0:
+            print(json.dumps({"profile_run": True, "workload": CFG.name, "decode_steps": DECODE,
+                              "value": value, "unit": "tok/s", "ttft_ms": statistics.median(ttft)}), flush=True)
+        model.close()
+        return 0
 
     # roofline of the dominant kernel (gate/up + SwiGLU GEMV), timed live with CUDA events
     model.reset()
@@ -302,6 +316,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--quick", action="store_true", help="profiling run: timed requests only")
+    ap.add_argument("--decode-steps", type=int, default=0, help="profiling run: decode steps per request")
+    ap.add_argument("--layers", type=int, default=0, help="profiling run: fewer layers (small ncu case)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)

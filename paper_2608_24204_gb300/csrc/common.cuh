@@ -99,6 +99,14 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
         : "memory");
 }
 
+// same without a cache hint (data that should stay in L2, e.g. the KV cache)
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
 // L2 policy for data read exactly once per step (weights): evict first.
 __device__ __forceinline__ uint64_t l2_evict_first() {
     uint64_t p;

@@ -1,7 +1,10 @@
 // Device buffers and the enqueue functions of the decode and prefill paths.
 #pragma once
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+
+#include <vector>
 
 #include "plan.h"
 
@@ -19,16 +22,25 @@ struct Bufs {
     float *m;         // decode SwiGLU output                               [F]
     float *logits;    // last logits                                        [V]
     int2 *amax;       // per-CTA argmax partials (value bits, index)        [num_sms]
-    float *attn;      // flash-decode partials [nkv][splits][group][d + 2]
     float2 *rope;     // (cos, sin) of p * theta^(-2i/d)                     [max_tokens][d/2]
     int *pages;       // logical -> physical KV page                         [max_pages]
     int *tok;         // prefill chunk tokens                                [max_chunk]
     float *X;         // prefill residual stream                             [max_chunk][H]
-    float *A;         // prefill GEMM input rows (fp32)                      [max_chunk][max(H,F,qdim)]
     float *Q;         // prefill queries after RoPE                          [max_chunk][qdim]
-    float *O;         // prefill attention output                            [max_chunk][qdim]
-    float *M;         // prefill SwiGLU output                               [max_chunk][F]
+    // prefill GEMM operands, each an fp32 activation split as hi + lo (bf16 bits)
+    uint16_t *Ahi, *Alo;  // RMSNorm output                                   [max_chunk][H]
+    uint16_t *Ohi, *Olo;  // attention output                                 [max_chunk][qdim]
+    uint16_t *Mhi, *Mlo;  // SwiGLU output                                    [max_chunk][F]
 };
+
+// TMA descriptors of the prefill GEMM operands (built once per context).
+struct PrefillMaps {
+    CUtensorMap ahi, alo, ohi, olo, mhi, mlo;          // activations, 128-row boxes
+    std::vector<CUtensorMap> wqkv, wo, wgu, wd;        // per layer weights, 256-row boxes
+};
+
+// Encodes every tensor map of `m`; returns an error message or nullptr.
+const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m);
 
 // Called around every launch when profiling (eager mode).
 struct LaunchHook {
@@ -53,8 +65,8 @@ cudaError_t enqueue_lm_head(const Plan &p, const Bufs &b, cudaStream_t st, bool 
 // Prefill of the chunk b.tok[0..T) at positions P..P+T-1 through every layer.
 // With lm_pos_add > 0 it then copies the chunk's last row to b.x and runs the
 // LM head, which advances ctrl[CTRL_POS] by lm_pos_add.
-cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, cudaStream_t st, int P, int T,
-                                  int lm_pos_add, LaunchHook *hook);
+cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMaps &maps,
+                                  cudaStream_t st, int P, int T, int lm_pos_add, LaunchHook *hook);
 
 // RoPE table for positions [0, max_tokens).
 cudaError_t enqueue_rope_table(const Plan &p, const Bufs &b, cudaStream_t st);

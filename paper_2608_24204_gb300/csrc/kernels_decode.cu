@@ -23,6 +23,8 @@ enum : int { SITE_GEMV_EMPTY = 11, SITE_GEMV_FULL = 12, SITE_GEMV_DRAIN = 13, SI
 struct GemvIn {
     const uint16_t *W;      // rows of this matrix, [n_units * rpu][K]
     int K, n_units, rpu, ups;
+    int stages;             // ring slots (<= kGemvMaxStages)
+    uint32_t slot_bytes;    // bytes per ring slot (>= ups * rpu * K * 2, multiple of 128)
     const float *in;        // input vector (x when gain != nullptr)
     const uint16_t *gain;   // RMSNorm gain (bf16) or nullptr for a plain input
     const uint16_t *embed;  // non-null: the input is embed[ctrl[CTRL_TOKEN]] (layer 0)
@@ -117,51 +119,90 @@ __device__ __forceinline__ bool better(float av, int ai, float bv, int bi) {
     return av > bv || (av == bv && ai < bi);
 }
 
-__device__ __forceinline__ void consumer_bar() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
-__device__ __forceinline__ float dot8(const uint4 w, const float *h) {
-    float s = bf16lo(w.x) * h[0];
-    s = fmaf(bf16hi(w.x), h[1], s);
-    s = fmaf(bf16lo(w.y), h[2], s);
-    s = fmaf(bf16hi(w.y), h[3], s);
-    s = fmaf(bf16lo(w.z), h[4], s);
-    s = fmaf(bf16hi(w.z), h[5], s);
-    s = fmaf(bf16lo(w.w), h[6], s);
-    s = fmaf(bf16hi(w.w), h[7], s);
-    return s;
+constexpr int kRedRows = 128;  // rows of partial sums per reduction batch
+constexpr int kGemvMaxStages = 8;
+// dynamic shared memory: [reduction scratch 2 x 8 warps x kRedRows fp32][ring]
+constexpr size_t kGemvRedBytes = 2 * 8 * kRedRows * 4;
+static inline size_t gemv_smem_bytes(int stages, uint32_t slot_bytes) {
+    return kGemvRedBytes + (size_t)stages * slot_bytes;
 }
 
-constexpr size_t kGemvSmem =
-    (size_t)kGemvStages * kGemvStageMax + 2 * kGemvStages * 8 + 2 * 8 * kGemvMaxRows * 4;
+// ------------------------------------------------------------------- GEMV ----
+// Grid: num_sms CTAs, each owning a contiguous, balanced range of units.  Each
+// consumer thread holds NCH 8-element chunks of the input vector in registers
+// (chunk c = tid + 256 j) and, for every row of a stage, contributes the dot
+// product over its chunks; warp sums go to shared memory and are reduced over
+// the 8 warps (fixed order) once per batch of up to kRedRows rows.
+// Shapes: every slot holds RPS rows (RPS a power of two, at most 8, RPS x K x 2
+// <= 32 KB, a multiple of the unit); consumer thread t covers the 8-element
+// chunks c = t + 256 j, j < NCH; FULL when the chunks cover K exactly (no tail
+// check in the inner loop).
+__host__ __device__ constexpr int gemv_rps(int K) {
+    return 2 * K * 8 <= 32768 ? 8 : 2 * K * 4 <= 32768 ? 4 : 2 * K * 2 <= 32768 ? 2 : 1;
+}
+__host__ __device__ constexpr int gemv_nch(int K) { return (K / 8 + 255) / 256; }
+
+constexpr int kGemvConsumers = 256;
+constexpr int kGemvWarps = 8;
+
+__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+    uint4 r;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "r"(addr));
+    return r;
+}
+
+// a + (8 bf16 weights) . (8 fp32 inputs)
+__device__ __forceinline__ float dot8(const uint4 w, const float *h, float a) {
+    a = fmaf(bf16lo(w.x), h[0], a);
+    a = fmaf(bf16hi(w.x), h[1], a);
+    a = fmaf(bf16lo(w.y), h[2], a);
+    a = fmaf(bf16hi(w.y), h[3], a);
+    a = fmaf(bf16lo(w.z), h[4], a);
+    a = fmaf(bf16hi(w.z), h[5], a);
+    a = fmaf(bf16lo(w.w), h[6], a);
+    a = fmaf(bf16hi(w.w), h[7], a);
+    return a;
+}
 
 // ------------------------------------------------------------------- GEMV ----
-// Grid: num_sms CTAs, each owning a contiguous, balanced range of units.
-template <int NCH, class Epi>
+// Grid: num_sms CTAs, each owning a contiguous, balanced range of units.  The
+// producer warp streams the CTA's rows, RPS per slot, through the ring; each of
+// the 8 consumer warps adds its chunks of every row and reduces the slot's RPS
+// rows with interleaved butterflies; warp sums go to shared memory and are
+// reduced over the warps (fixed order) once per kRedRows rows, then passed to
+// the epilogue.
+template <int NCH, int RPS, bool FULL, class Epi>
 __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const GemvIn g, const Epi epi_in) {
     extern __shared__ __align__(128) uint8_t smem[];
-    uint8_t *ring = smem;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kGemvStages * kGemvStageMax);
-    float *red = reinterpret_cast<float *>(bars + 2 * kGemvStages);  // [2][8][kGemvMaxRows]
-    __shared__ float s_part[8];
+    float *red = reinterpret_cast<float *>(smem);  // [2][kGemvWarps][kRedRows]
+    uint8_t *ring = smem + kGemvRedBytes;
+    __shared__ __align__(8) uint64_t bars[2 * kGemvMaxStages];  // full[S], empty[S]
+    __shared__ float s_part[kGemvWarps];
     __shared__ int s_abort;
-    __shared__ float s_bv[8];
-    __shared__ int s_bi[8];
+    __shared__ float s_bv[kGemvWarps];
+    __shared__ int s_bi[kGemvWarps];
     __shared__ int s_last;
+    const int S = g.stages;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = gridDim.x;
     const int u0 = (int)(((long long)blockIdx.x * g.n_units) / G);
     const int u1 = (int)(((long long)(blockIdx.x + 1) * g.n_units) / G);
     const int nunits = u1 - u0;
-    const int nst = (nunits + g.ups - 1) / g.ups;
-    const uint32_t unit_bytes = (uint32_t)g.rpu * (uint32_t)g.K * 2u;
+    const int total_rows = nunits * g.rpu;
+    const int nst = (total_rows + RPS - 1) / RPS;
     int *err = g.ctrl + CTRL_ERR;
 
-    const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kGemvStages);
+    const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kGemvMaxStages);
     if (tid == 0) {
-        for (int s = 0; s < kGemvStages; ++s) {
+        for (int s = 0; s < S; ++s) {
             mbar_init(full0 + 8 * s, 1);
-            mbar_init(empty0 + 8 * s, 8);
+            mbar_init(empty0 + 8 * s, kGemvWarps);
         }
         fence_barrier_init();
         s_abort = 0;
@@ -169,26 +210,24 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const GemvIn g, c
     __syncthreads();
     griddep_launch_dependents();
 
-    if (warp == 8) {  // ------------------------------------------ producer
+    if (warp == kGemvWarps) {  // ------------------------------------ producer
         if (lane == 0) {
             const uint64_t pol = l2_evict_first();
             const uint32_t ring0 = smem_u32(ring);
+            const uint16_t *src = g.W + (size_t)u0 * g.rpu * g.K;
             int issued = 0;
             for (int s = 0; s < nst; ++s) {
-                const int slot = s % kGemvStages;
-                if (s >= kGemvStages &&
-                    !mbar_wait(empty0 + 8 * slot, ((s / kGemvStages) + 1) & 1, err, SITE_GEMV_EMPTY))
-                    break;
-                const int un = min(g.ups, nunits - s * g.ups);
-                const uint32_t bytes = (uint32_t)un * unit_bytes;
+                const int slot = s % S;
+                if (s >= S && !mbar_wait(empty0 + 8 * slot, ((s / S) + 1) & 1, err, SITE_GEMV_EMPTY)) break;
+                const int rows = min(RPS, total_rows - s * RPS);
+                const uint32_t bytes = (uint32_t)rows * (uint32_t)g.K * 2u;
                 mbar_arrive_expect_tx(full0 + 8 * slot, bytes);
-                bulk_g2s(ring0 + slot * kGemvStageMax,
-                         g.W + (size_t)(u0 + s * g.ups) * g.rpu * g.K, bytes, full0 + 8 * slot, pol);
+                bulk_g2s(ring0 + slot * g.slot_bytes, src + (size_t)s * RPS * g.K, bytes, full0 + 8 * slot, pol);
                 issued = s + 1;
             }
             // no copy may still be landing in this CTA's shared memory when it exits
-            for (int s = max(0, issued - kGemvStages); s < issued; ++s)
-                mbar_wait(full0 + 8 * (s % kGemvStages), (s / kGemvStages) & 1, err, SITE_GEMV_DRAIN);
+            for (int s = max(0, issued - S); s < issued; ++s)
+                mbar_wait(full0 + 8 * (s % S), (s / S) & 1, err, SITE_GEMV_DRAIN);
         }
         return;
     }
@@ -202,14 +241,12 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const GemvIn g, c
     const int tok = g.embed ? g.ctrl[CTRL_TOKEN] : 0;
 #pragma unroll
     for (int j = 0; j < NCH; ++j) {
-        const int c = tid + 256 * j;
-        if (c < nchunks) {
+        const int c = tid + kGemvConsumers * j;
+        if (FULL || c < nchunks) {
             if (g.embed) {
                 const uint4 w = *reinterpret_cast<const uint4 *>(g.embed + (size_t)tok * g.K + c * 8);
-                h[j][0] = bf16lo(w.x); h[j][1] = bf16hi(w.x);
-                h[j][2] = bf16lo(w.y); h[j][3] = bf16hi(w.y);
-                h[j][4] = bf16lo(w.z); h[j][5] = bf16hi(w.z);
-                h[j][6] = bf16lo(w.w); h[j][7] = bf16hi(w.w);
+                h[j][0] = bf16lo(w.x); h[j][1] = bf16hi(w.x); h[j][2] = bf16lo(w.y); h[j][3] = bf16hi(w.y);
+                h[j][4] = bf16lo(w.z); h[j][5] = bf16hi(w.z); h[j][6] = bf16lo(w.w); h[j][7] = bf16hi(w.w);
                 if (blockIdx.x == 0) {
                     float4 *dst = reinterpret_cast<float4 *>(g.x_out + c * 8);
                     dst[0] = make_float4(h[j][0], h[j][1], h[j][2], h[j][3]);
@@ -231,15 +268,15 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const GemvIn g, c
     if (g.gain) {  // RMSNorm prologue: every CTA reduces the whole vector in the same order
         ss = warp_sum(ss);
         if (lane == 0) s_part[warp] = ss;
-        consumer_bar();
+        consumer_sync();
         float tot = 0.f;
 #pragma unroll
-        for (int w = 0; w < 8; ++w) tot += s_part[w];
+        for (int w = 0; w < kGemvWarps; ++w) tot += s_part[w];
         const float rinv = 1.0f / sqrtf(tot / (float)g.K + g.eps);
 #pragma unroll
         for (int j = 0; j < NCH; ++j) {
-            const int c = tid + 256 * j;
-            if (c < nchunks) {
+            const int c = tid + kGemvConsumers * j;
+            if (FULL || c < nchunks) {
                 const uint4 gw = *reinterpret_cast<const uint4 *>(g.gain + c * 8);
                 const float gg[8] = {bf16lo(gw.x), bf16hi(gw.x), bf16lo(gw.y), bf16hi(gw.y),
                                      bf16lo(gw.z), bf16hi(gw.z), bf16lo(gw.w), bf16hi(gw.w)};
@@ -249,43 +286,75 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const GemvIn g, c
         }
     }
 
-    int buf = 0;
+    const uint32_t row_bytes = (uint32_t)g.K * 2u;
+    const uint32_t my0 = smem_u32(ring) + (uint32_t)tid * 16u;   // this thread's chunk 0 in slot 0
+    const bool tail_ok = FULL || tid + kGemvConsumers * (NCH - 1) < nchunks;
+    int buf = 0, brow = 0, bunit0 = 0, slot = 0;
+    uint32_t phase = 0;
+    bool ok = true;
     for (int s = 0; s < nst; ++s) {
-        const int slot = s % kGemvStages;
-        const int un = min(g.ups, nunits - s * g.ups);
-        const int rows = un * g.rpu;
-        const bool ok = mbar_wait(full0 + 8 * slot, (s / kGemvStages) & 1, err, SITE_GEMV_FULL);
+        const int rows = min(RPS, total_rows - s * RPS);
+        ok = ok && !*reinterpret_cast<volatile int *>(&s_abort) &&
+             mbar_wait(full0 + 8 * slot, phase, err, SITE_GEMV_FULL);
         if (!ok) s_abort = 1;
-        if (ok) {
-            const uint8_t *st = ring + (size_t)slot * kGemvStageMax;
-            float *rb = red + (size_t)(buf * 8 + warp) * kGemvMaxRows;
-            for (int r = 0; r < rows; ++r) {
-                const uint8_t *row = st + (size_t)r * g.K * 2;
-                float acc = 0.f;
+        float acc[RPS];
 #pragma unroll
-                for (int j = 0; j < NCH; ++j) {
-                    const int c = tid + 256 * j;
-                    if (c < nchunks) acc += dot8(*reinterpret_cast<const uint4 *>(row + c * 16), h[j]);
-                }
-                acc = warp_sum(acc);
-                if (lane == 0) rb[r] = acc;
+        for (int r = 0; r < RPS; ++r) acc[r] = 0.f;
+        if (ok) {
+            const uint32_t sb = my0 + (uint32_t)slot * g.slot_bytes;
+            if (rows == RPS) {
+#pragma unroll
+                for (int r = 0; r < RPS; ++r)
+#pragma unroll
+                    for (int j = 0; j < NCH; ++j)
+                        if (j < NCH - 1 || tail_ok)
+                            acc[r] = dot8(lds128(sb + r * row_bytes + j * kGemvConsumers * 16), h[j], acc[r]);
+            } else {   // the CTA's last slot may hold fewer rows
+#pragma unroll
+                for (int r = 0; r < RPS; ++r)
+                    if (r < rows)
+#pragma unroll
+                        for (int j = 0; j < NCH; ++j)
+                            if (j < NCH - 1 || tail_ok)
+                                acc[r] = dot8(lds128(sb + r * row_bytes + j * kGemvConsumers * 16), h[j], acc[r]);
             }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(empty0 + 8 * slot);
-        consumer_bar();
-        if (s_abort) break;
-        if (tid < un) {
-            float v[2];
-            for (int j = 0; j < g.rpu; ++j) {
-                float t = 0.f;
-#pragma unroll
-                for (int w = 0; w < 8; ++w) t += red[(size_t)(buf * 8 + w) * kGemvMaxRows + tid * g.rpu + j];
-                v[j] = t;
-            }
-            epi.unit(u0 + s * g.ups + tid, v);
+        if (++slot == S) {
+            slot = 0;
+            phase ^= 1u;
         }
-        buf ^= 1;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+            for (int r = 0; r < RPS; ++r) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
+        if (lane == 0) {
+            float *rb = red + (size_t)(buf * kGemvWarps + warp) * kRedRows + brow;
+#pragma unroll
+            for (int r = 0; r < RPS; ++r)
+                if (r < rows) rb[r] = acc[r];
+        }
+        brow += rows;
+        if (s == nst - 1 || brow + RPS > kRedRows) {
+            consumer_sync();
+            if (s_abort) break;
+            const int bunits = brow / g.rpu;
+            for (int t = tid; t < bunits; t += kGemvConsumers) {
+                float v[2];
+                for (int j = 0; j < g.rpu; ++j) {
+                    float sum = 0.f;
+#pragma unroll
+                    for (int w = 0; w < kGemvWarps; ++w)
+                        sum += red[(size_t)(buf * kGemvWarps + w) * kRedRows + t * g.rpu + j];
+                    v[j] = sum;
+                }
+                epi.unit(u0 + bunit0 + t, v);
+            }
+            bunit0 += bunits;
+            brow = 0;
+            buf ^= 1;
+        }
     }
 
     if constexpr (Epi::kArgmax) {
@@ -299,16 +368,16 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const GemvIn g, c
             if (better(ov, oi, bv, bi)) { bv = ov; bi = oi; }
         }
         if (lane == 0) { s_bv[warp] = bv; s_bi[warp] = bi; }
-        consumer_bar();
+        consumer_sync();
         if (tid == 0) {
-            for (int w = 1; w < 8; ++w)
+            for (int w = 1; w < kGemvWarps; ++w)
                 if (better(s_bv[w], s_bi[w], bv, bi)) { bv = s_bv[w]; bi = s_bi[w]; }
             epi.partial[blockIdx.x] = make_int2(__float_as_int(bv), bi);
             __threadfence();
             const int t = atomicAdd(epi.ctrl + CTRL_LM_TICKET, 1);
             s_last = (t == G - 1);
         }
-        consumer_bar();
+        consumer_sync();
         if (s_last && tid == 0) {
             __threadfence();
             float fv = -INFINITY;
@@ -329,80 +398,156 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const GemvIn g, c
 }
 
 // ------------------------------------------------------------ flash-decode ----
-// Grid (splits, nkv); block = 32 * group threads, warp w = query head g*group+w.
-// Each CTA covers a contiguous range of KV pages of head g (length taken from the
-// device position, so one captured graph serves every step), keeps a warp-level
-// online softmax per query head, writes (m, l, acc[d]) partials, and the last
-// CTA of each KV head combines the partials in split order.
+// Grid (kFdSplits, nkv) in clusters of kFdSplits CTAs: one cluster per KV head g.
+// Block = 32 * (group + 1) threads: warp w < group is query head g*group+w, the
+// last warp streams this CTA's KV pages (K and V blocks of head g, 16 x d bf16
+// each, contiguous in a page) through a 4-stage TMA ring.  The length comes from
+// the device position, so one captured graph serves every step.  Each query
+// warp keeps an online softmax over its CTA's pages and leaves (m, l, acc[d]) in
+// shared memory; after a cluster barrier the CTA of rank 0 combines the
+// kFdSplits partials over distributed shared memory, in rank order.
+constexpr int kFdStages = 4;
+constexpr int kFdSplits = 16;   // cluster size (non-portable: 16 > 8)
+
 struct FDArgs {
     const float *q;
     const uint16_t *kv;  // this layer's pages
     const int *pages;
     int *ctrl;
-    float *part;
     float *o;
-    int nkv, group, splits;
+    int nkv, group;
     size_t page_elems;
     float qscale;        // log2(e) / sqrt(d)
 };
 
+enum : int { SITE_FD_EMPTY = 31, SITE_FD_FULL = 32, SITE_FD_DRAIN = 33 };
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t dsmem_addr(const void *local, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(local)), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ float ld_dsmem(uint32_t addr) {
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+    return v;
+}
+
 template <int D>
-__global__ void __launch_bounds__(256) flash_decode_kernel(const FDArgs a) {
+__global__ void __launch_bounds__(288) flash_decode_kernel(const FDArgs a) {
     constexpr int EPL = D / 32;
-    __shared__ int s_last;
+    constexpr uint32_t BLK = kPage * D * 2;     // bytes of one K (or V) block of a page
+    extern __shared__ __align__(128) uint8_t fsm[];   // [kFdStages][K block | V block]
+    __shared__ __align__(8) uint64_t full_bar[kFdStages], empty_bar[kFdStages];
+    __shared__ __align__(16) float s_part[8][D + 4];  // per query warp: acc[D], m, l
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = blockIdx.y, split = blockIdx.x;
-    const int head = g * a.group + w;
-    griddep_launch_dependents();
-    griddep_wait();
-
-    const int len = a.ctrl[CTRL_POS] + 1;
-    const int npages = (len + kPage - 1) / kPage;
-    const int pps = (npages + a.splits - 1) / a.splits;
-    const int p0 = split * pps, p1 = min(npages, p0 + pps);
-
-    float qv[EPL], acc[EPL];
-#pragma unroll
-    for (int e = 0; e < EPL; ++e) {
-        qv[e] = a.q[head * D + lane * EPL + e] * a.qscale;
-        acc[e] = 0.f;
+    const int g = blockIdx.y;
+    const uint32_t rank = cluster_ctarank();
+    int *err = a.ctrl + CTRL_ERR;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kFdStages; ++s) {
+            mbar_init(smem_u32(&full_bar[s]), 1);
+            mbar_init(smem_u32(&empty_bar[s]), a.group);
+        }
+        fence_barrier_init();
     }
-    float m = -INFINITY, l = 0.f;
-    for (int p = p0; p < p1; ++p) {
-        const uint16_t *Kb = a.kv + (size_t)a.pages[p] * a.page_elems + (size_t)g * kPage * D;
-        const uint16_t *Vb = Kb + (size_t)a.nkv * kPage * D;
-        const int ntok = min(kPage, len - p * kPage);
-        float sc[kPage];
-        float mx = m;
+    __syncthreads();
+    griddep_launch_dependents();
+
+    // the position is only advanced at the end of a step, so it is stable here
+    const int len = *reinterpret_cast<volatile int *>(a.ctrl + CTRL_POS) + 1;
+    const int npages = (len + kPage - 1) / kPage;
+    const int pps = (npages + kFdSplits - 1) / kFdSplits;
+    const int p0 = (int)rank * pps;
+    const int n = max(0, min(npages, p0 + pps) - p0);
+
+    if (w == a.group) {  // ---------------------------------------- producer
+        if (lane == 0) {
+            const uint32_t ring0 = smem_u32(fsm);
+            int issued = 0;
+            bool waited = false;
+            for (int i = 0; i < n; ++i) {
+                const int s = i % kFdStages;
+                if (i >= kFdStages &&
+                    !mbar_wait(smem_u32(&empty_bar[s]), ((i / kFdStages) + 1) & 1, err, SITE_FD_EMPTY))
+                    break;
+                // the page holding the current position is written by the preceding kernel
+                if (!waited && p0 + i == npages - 1) {
+                    griddep_wait();
+                    waited = true;
+                }
+                const uint16_t *Kb = a.kv + (size_t)a.pages[p0 + i] * a.page_elems + (size_t)g * kPage * D;
+                const uint16_t *Vb = Kb + (size_t)a.nkv * kPage * D;
+                const uint32_t fb = smem_u32(&full_bar[s]);
+                mbar_arrive_expect_tx(fb, 2 * BLK);
+                bulk_g2s(ring0 + s * 2 * BLK, Kb, BLK, fb);
+                bulk_g2s(ring0 + s * 2 * BLK + BLK, Vb, BLK, fb);
+                issued = i + 1;
+            }
+            for (int i = max(0, issued - kFdStages); i < issued; ++i)
+                mbar_wait(smem_u32(&full_bar[i % kFdStages]), (i / kFdStages) & 1, err, SITE_FD_DRAIN);
+        }
+        __syncwarp();
+    } else {  // ------------------------------------------------- query warps
+        griddep_wait();
+        const int head = g * a.group + w;
+        float qv[EPL], acc[EPL];
 #pragma unroll
-        for (int t = 0; t < kPage; ++t) {
-            float s = -INFINITY;
-            if (t < ntok) {
-                const uint16_t *kr = Kb + t * D + lane * EPL;
-                float part = 0.f;
+        for (int e = 0; e < EPL; ++e) {
+            qv[e] = a.q[head * D + lane * EPL + e] * a.qscale;
+            acc[e] = 0.f;
+        }
+        float m = -INFINITY, l = 0.f;
+        bool ok = true;
+        for (int i = 0; i < n && ok; ++i) {
+            const int s = i % kFdStages;
+            ok = mbar_wait(smem_u32(&full_bar[s]), (i / kFdStages) & 1, err, SITE_FD_FULL);
+            if (!ok) break;
+            const uint8_t *Ks = fsm + (size_t)s * 2 * BLK;
+            const uint8_t *Vs = Ks + BLK;
+            const int ntok = min(kPage, len - (p0 + i) * kPage);
+            float sc[kPage];
+#pragma unroll
+            for (int t = 0; t < kPage; ++t) {
+                const uint8_t *kr = Ks + (t * D + lane * EPL) * 2;
                 if constexpr (EPL == 4) {
                     const uint2 kw = *reinterpret_cast<const uint2 *>(kr);
-                    part = qv[0] * bf16lo(kw.x) + qv[1] * bf16hi(kw.x) + qv[2] * bf16lo(kw.y) +
-                           qv[3] * bf16hi(kw.y);
+                    sc[t] = qv[0] * bf16lo(kw.x) + qv[1] * bf16hi(kw.x) + qv[2] * bf16lo(kw.y) +
+                            qv[3] * bf16hi(kw.y);
                 } else {
                     const uint32_t kw = *reinterpret_cast<const uint32_t *>(kr);
-                    part = qv[0] * bf16lo(kw) + qv[1] * bf16hi(kw);
+                    sc[t] = qv[0] * bf16lo(kw) + qv[1] * bf16hi(kw);
                 }
-                s = warp_sum(part);
             }
-            sc[t] = s;
-            mx = fmaxf(mx, s);
-        }
-        const float corr = exp2f(m - mx);
-        l *= corr;
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) acc[e] *= corr;
+            for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
-        for (int t = 0; t < kPage; ++t) {
-            if (t < ntok) {
+                for (int t = 0; t < kPage; ++t) sc[t] += __shfl_xor_sync(0xffffffffu, sc[t], o);
+            float mx = m;
+#pragma unroll
+            for (int t = 0; t < kPage; ++t) {
+                if (t >= ntok) sc[t] = -INFINITY;
+                mx = fmaxf(mx, sc[t]);
+            }
+            const float corr = exp2f(m - mx);
+            l *= corr;
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) acc[e] *= corr;
+#pragma unroll
+            for (int t = 0; t < kPage; ++t) {
+                // slots past the length are never read: unwritten cache memory may hold NaN bits
+                if (t >= ntok) break;
                 const float pt = exp2f(sc[t] - mx);
                 l += pt;
-                const uint16_t *vr = Vb + t * D + lane * EPL;
+                const uint8_t *vr = Vs + (t * D + lane * EPL) * 2;
                 if constexpr (EPL == 4) {
                     const uint2 vw = *reinterpret_cast<const uint2 *>(vr);
                     acc[0] = fmaf(pt, bf16lo(vw.x), acc[0]);
@@ -415,44 +560,43 @@ __global__ void __launch_bounds__(256) flash_decode_kernel(const FDArgs a) {
                     acc[1] = fmaf(pt, bf16hi(vw), acc[1]);
                 }
             }
+            m = mx;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[s]));
         }
-        m = mx;
-    }
-    float *pp = a.part + ((size_t)(g * a.splits + split) * a.group + w) * (D + 2);
 #pragma unroll
-    for (int e = 0; e < EPL; ++e) pp[lane * EPL + e] = acc[e];
-    if (lane == 0) {
-        pp[D] = m;
-        pp[D + 1] = l;
+        for (int e = 0; e < EPL; ++e) s_part[w][lane * EPL + e] = acc[e];
+        if (lane == 0) {
+            s_part[w][D] = m;
+            s_part[w][D + 1] = l;
+        }
     }
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        const int t = atomicAdd(a.ctrl + CTRL_ATTN_TICKET0 + g, 1);
-        s_last = (t == a.splits - 1);
-    }
-    __syncthreads();
-    if (!s_last) return;
-    __threadfence();
-    float M = -INFINITY;
-    for (int s = 0; s < a.splits; ++s) {
-        const float *ps = a.part + ((size_t)(g * a.splits + s) * a.group + w) * (D + 2);
-        M = fmaxf(M, __ldcg(ps + D));
-    }
-    float L = 0.f, out[EPL];
+    cluster_sync_all();   // every CTA's partials are written and visible to the cluster
+    if (rank == 0 && w < a.group) {
+        const int head = g * a.group + w;
+        float ms = -INFINITY, ls = 0.f;
+        if (lane < kFdSplits) {
+            ms = ld_dsmem(dsmem_addr(&s_part[w][D], lane));
+            ls = ld_dsmem(dsmem_addr(&s_part[w][D + 1], lane));
+        }
+        const float M = warp_max(ms);
+        const float f = lane < kFdSplits ? exp2f(ms - M) : 0.f;   // empty splits: exp2(-inf) = 0
+        const float L = warp_sum(ls * f);
+        float out[EPL];
 #pragma unroll
-    for (int e = 0; e < EPL; ++e) out[e] = 0.f;
-    for (int s = 0; s < a.splits; ++s) {
-        const float *ps = a.part + ((size_t)(g * a.splits + s) * a.group + w) * (D + 2);
-        const float f = exp2f(__ldcg(ps + D) - M);
-        L = fmaf(__ldcg(ps + D + 1), f, L);
+        for (int e = 0; e < EPL; ++e) out[e] = 0.f;
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) out[e] = fmaf(__ldcg(ps + lane * EPL + e), f, out[e]);
+        for (int s = 0; s < kFdSplits; ++s) {
+            const float fs = __shfl_sync(0xffffffffu, f, s);
+            const uint32_t ra = dsmem_addr(&s_part[w][lane * EPL], (uint32_t)s);
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) out[e] = fmaf(ld_dsmem(ra + 4 * e), fs, out[e]);
+        }
+        const float inv = 1.0f / L;
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) a.o[head * D + lane * EPL + e] = out[e] * inv;
     }
-    const float inv = 1.0f / L;
-#pragma unroll
-    for (int e = 0; e < EPL; ++e) a.o[head * D + lane * EPL + e] = out[e] * inv;
-    if (threadIdx.x == 0) a.ctrl[CTRL_ATTN_TICKET0 + g] = 0;
+    cluster_sync_all();   // keep every CTA's shared memory alive until rank 0 has read it
 }
 
 // ------------------------------------------------------------ probe kernel ----
@@ -484,33 +628,64 @@ static cudaError_t launch(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStr
     return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
+template <int D>
+static cudaError_t launch_fd(const Plan &p, const FDArgs &fa, cudaStream_t st, bool pdl) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kFdSplits, p.nkv);
+    cfg.blockDim = dim3(32 * (p.group + 1));
+    cfg.dynamicSmemBytes = (size_t)kFdStages * 2 * kPage * D * 2;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = kFdSplits;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, flash_decode_kernel<D>, fa);
+}
+
+// the (NCH, RPS, FULL) shapes of every supported K (K % 8 == 0, K <= 16384)
+#define WICI_GEMV_SHAPES(X)                                                                     \
+    X(1, 8, true) X(1, 8, false) X(2, 4, true) X(2, 4, false) X(3, 2, true) X(3, 2, false)     \
+    X(4, 2, true) X(4, 2, false) X(5, 1, true) X(5, 1, false) X(6, 1, true) X(6, 1, false)     \
+    X(7, 1, true) X(7, 1, false) X(8, 1, true) X(8, 1, false)
+
 template <class Epi>
-static void *gemv_fn(int nch) {
-    switch (nch) {
-        case 1: return (void *)gemv_kernel<1, Epi>;
-        case 2: return (void *)gemv_kernel<2, Epi>;
-        case 3: return (void *)gemv_kernel<3, Epi>;
-        case 4: return (void *)gemv_kernel<4, Epi>;
-        case 5: return (void *)gemv_kernel<5, Epi>;
-        case 6: return (void *)gemv_kernel<6, Epi>;
-        case 7: return (void *)gemv_kernel<7, Epi>;
-        case 8: return (void *)gemv_kernel<8, Epi>;
-    }
+static void *gemv_fn(int K) {
+    const int nch = gemv_nch(K), rps = gemv_rps(K);
+    const bool full = (K / 8) == nch * kGemvConsumers;
+#define WICI_PICK(N, R, F) \
+    if (nch == N && rps == R && full == F) return (void *)gemv_kernel<N, R, F, Epi>;
+    WICI_GEMV_SHAPES(WICI_PICK)
+#undef WICI_PICK
     return nullptr;
 }
 
 template <class Epi>
 static cudaError_t set_gemv_attrs() {
-    for (int n = 1; n <= 8; ++n) {
-        cudaError_t e = cudaFuncSetAttribute(gemv_fn<Epi>(n), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)kGemvSmem);
-        if (e != cudaSuccess) return e;
+#define WICI_ATTR(N, R, F)                                                                              \
+    {                                                                                                   \
+        cudaError_t e = cudaFuncSetAttribute(gemv_kernel<N, R, F, Epi>,                                \
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,              \
+                                             (int)gemv_smem_bytes(1, kGemvRingBytes));                 \
+        if (e != cudaSuccess) return e;                                                                 \
     }
+    WICI_GEMV_SHAPES(WICI_ATTR)
+#undef WICI_ATTR
     return cudaSuccess;
 }
 
 cudaError_t setup_kernels() {
     cudaError_t e;
+    if ((e = cudaFuncSetAttribute(flash_decode_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
+        cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(flash_decode_kernel<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
+        cudaSuccess)
+        return e;
     if ((e = set_gemv_attrs<EpiResidual>()) != cudaSuccess) return e;
     if ((e = set_gemv_attrs<EpiSwiGLU>()) != cudaSuccess) return e;
     if ((e = set_gemv_attrs<EpiQKV>()) != cudaSuccess) return e;
@@ -518,25 +693,26 @@ cudaError_t setup_kernels() {
     return cudaSuccess;
 }
 
-// units per stage: as many whole units as fit one stage, at most kGemvMaxRows rows
-static int units_per_stage(int K, int rpu) {
-    const int unit_bytes = rpu * K * 2;
-    int ups = (int)(kGemvStageMax / (uint32_t)unit_bytes);
-    ups = ups < 1 ? 1 : ups;
-    while (ups * rpu > kGemvMaxRows) --ups;
-    return ups;
+// Ring geometry: slots of gemv_rps(K) rows, as many as fit kGemvRingBytes (2 to 8).
+static void ring_geometry(GemvIn &g) {
+    const int rps = gemv_rps(g.K);
+    g.ups = rps / g.rpu;
+    g.slot_bytes = ((uint32_t)rps * (uint32_t)g.K * 2u + 127u) & ~127u;
+    int st = (int)(kGemvRingBytes / g.slot_bytes);
+    g.stages = st < 2 ? 2 : (st > kGemvMaxStages ? kGemvMaxStages : st);
 }
 
 template <class Epi>
 static cudaError_t launch_gemv(const Plan &p, GemvIn g, Epi epi, cudaStream_t st, bool pdl,
                                LaunchHook *hook, const char *name) {
-    g.ups = units_per_stage(g.K, g.rpu);
-    const int nch = (g.K / 8 + 255) / 256;
-    if (nch < 1 || nch > 8) return cudaErrorInvalidValue;
-    const int grid = p.num_sms;
+    ring_geometry(g);
+    void *fn = gemv_fn<Epi>(g.K);
+    if (!fn || g.ups < 1) return cudaErrorInvalidValue;
+    const int grid = p.num_sms * kGemvCtasPerSm;
     if (hook) hook->before(name);
-    cudaError_t e = launch(reinterpret_cast<void (*)(const GemvIn, const Epi)>(gemv_fn<Epi>(nch)),
-                           dim3(grid), dim3(kGemvThreads), kGemvSmem, st, pdl, g, epi);
+    cudaError_t e = launch(reinterpret_cast<void (*)(const GemvIn, const Epi)>(fn),
+                           dim3(grid), dim3(kGemvThreads), gemv_smem_bytes(g.stages, g.slot_bytes), st, pdl,
+                           g, epi);
     if (hook) hook->after(name);
     return e;
 }
@@ -596,15 +772,12 @@ cudaError_t enqueue_decode_step(const Plan &p, const Bufs &b, cudaStream_t st, b
         eq.page_elems = p.kv_page_elems;
         if ((e = launch_gemv(p, g, eq, st, pdl && l > 0, hook, "qkv_rope_kvappend")) != cudaSuccess) return e;
         // A5: attention
-        FDArgs fa = {b.q, kvl, b.pages, b.ctrl, b.attn, b.o, p.nkv, p.group, p.attn_splits,
-                     p.kv_page_elems, qscale};
+        FDArgs fa = {b.q, kvl, b.pages, b.ctrl, b.o, p.nkv, p.group, p.kv_page_elems, qscale};
         if (hook) hook->before("flash_decode");
         if (p.d == 128)
-            e = launch(flash_decode_kernel<128>, dim3(p.attn_splits, p.nkv), dim3(32 * p.group), 0, st,
-                       pdl, fa);
+            e = launch_fd<128>(p, fa, st, pdl);
         else
-            e = launch(flash_decode_kernel<64>, dim3(p.attn_splits, p.nkv), dim3(32 * p.group), 0, st,
-                       pdl, fa);
+            e = launch_fd<64>(p, fa, st, pdl);
         if (hook) hook->after("flash_decode");
         if (e != cudaSuccess) return e;
         // A6: O projection + residual

@@ -1,14 +1,24 @@
-// Prefill kernels: a chunk of T prompt tokens at positions P..P+T-1 through
-// every layer, fp32 activations.  The matrix products here are CUDA-core
-// tiled GEMMs with fused epilogues (RoPE + KV append, residual add, SwiGLU).
+// Prefill: a chunk of T prompt tokens at positions P..P+T-1 through every
+// layer.  The four linear maps of a layer run on the tcgen05 GEMM (gemm_tc.cuh)
+// with fused epilogues (bias + RoPE + paged KV append, residual add, SwiGLU);
+// the kernels around them produce the GEMM operands as bf16 hi/lo pairs.
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
 
 #include "common.cuh"
+#include "gemm_tc.cuh"
 #include "kernels.h"
 
 namespace wici {
+
+// a = hi + lo with hi = bf16(a), lo = bf16(a - hi)
+__device__ __forceinline__ void split_store(uint16_t *hi, uint16_t *lo, size_t i, float a) {
+    const uint16_t h = f32_to_bf16(a);
+    hi[i] = h;
+    lo[i] = f32_to_bf16(a - bf16_to_f32(h));
+}
 
 // ----------------------------------------------------------- embed / norm ----
 __global__ void embed_rows_kernel(const uint16_t *E, const int *tok, float *X, int H) {
@@ -17,8 +27,9 @@ __global__ void embed_rows_kernel(const uint16_t *E, const int *tok, float *X, i
     for (int i = threadIdx.x; i < H; i += blockDim.x) X[(size_t)t * H + i] = bf16_to_f32(row[i]);
 }
 
-// A[t] = X[t] / sqrt(mean(X[t]^2) + eps) * g
-__global__ void rmsnorm_rows_kernel(const float *X, const uint16_t *g, float *A, int H, float eps) {
+// A[t] = X[t] / sqrt(mean(X[t]^2) + eps) * g, stored as a hi/lo bf16 pair
+__global__ void rmsnorm_rows_kernel(const float *X, const uint16_t *g, uint16_t *Ahi, uint16_t *Alo, int H,
+                                    float eps) {
     __shared__ float s_part[32];
     const int t = blockIdx.x;
     const float *x = X + (size_t)t * H;
@@ -31,11 +42,11 @@ __global__ void rmsnorm_rows_kernel(const float *X, const uint16_t *g, float *A,
     for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += s_part[w];
     const float rinv = 1.0f / sqrtf(tot / (float)H + eps);
     for (int i = threadIdx.x; i < H; i += blockDim.x)
-        A[(size_t)t * H + i] = x[i] * rinv * bf16_to_f32(g[i]);
+        split_store(Ahi, Alo, (size_t)t * H + i, x[i] * rinv * bf16_to_f32(g[i]));
 }
 
 // --------------------------------------------------------------- epilogues ----
-// unit(t, c, v): row t, output columns (c, c+1) with values v[0], v[1]
+// pair(t, c, a, b): GEMM output row t, columns (c, c + 1)
 struct PEpiQKV {  // packed QKV columns -> Q (fp32) and K/V pages (bf16)
     float *Q;
     uint16_t *kv;
@@ -79,76 +90,29 @@ struct PEpiResidual {  // X[t][c] += v
     float *X;
     int ld;
     __device__ void pair(int t, int c, float a, float b) const {
-        X[(size_t)t * ld + c] += a;
-        X[(size_t)t * ld + c + 1] += b;
+        float2 *p = reinterpret_cast<float2 *>(X + (size_t)t * ld + c);
+        float2 v = *p;
+        v.x += a;
+        v.y += b;
+        *p = v;
     }
 };
 
-struct PEpiSwiGLU {  // interleaved (gate, up) columns -> M[t][c/2] = silu(g) * u
-    float *M;
+struct PEpiSwiGLU {  // interleaved (gate, up) columns -> M[t][c/2] = silu(g) * u as hi/lo
+    uint16_t *Mhi, *Mlo;
     int ld;
     __device__ void pair(int t, int c, float a, float b) const {
-        M[(size_t)t * ld + (c >> 1)] = a / (1.0f + expf(-a)) * b;
+        split_store(Mhi, Mlo, (size_t)t * ld + (c >> 1), a / (1.0f + expf(-a)) * b);
     }
 };
-
-// ---------------------------------------------------------------- GEMM ------
-// C[T][N] = A[T][K] (fp32) . W[N][K]^T (bf16), fp32 accumulation.
-// 64x64 output tile, 256 threads, 4x4 outputs per thread.
-constexpr int GBM = 64, GBN = 64, GBK = 16;
-
-template <class Epi>
-__global__ void __launch_bounds__(256) gemm_simt_kernel(const float *A, const uint16_t *W, int T,
-                                                        int N, int K, const Epi epi) {
-    __shared__ float As[GBK][GBM + 4];
-    __shared__ float Ws[GBK][GBN + 4];
-    const int tid = threadIdx.x;
-    const int tx = tid & 15, ty = tid >> 4;
-    const int m0 = blockIdx.y * GBM, n0 = blockIdx.x * GBN;
-    float acc[4][4] = {};
-    for (int k0 = 0; k0 < K; k0 += GBK) {
-        for (int i = tid; i < GBM * GBK; i += 256) {
-            const int r = i / GBK, k = i % GBK;
-            const int gm = m0 + r, gk = k0 + k;
-            As[k][r] = (gm < T && gk < K) ? A[(size_t)gm * K + gk] : 0.f;
-            const int gn = n0 + r;
-            Ws[k][r] = (gn < N && gk < K) ? bf16_to_f32(W[(size_t)gn * K + gk]) : 0.f;
-        }
-        __syncthreads();
-#pragma unroll
-        for (int k = 0; k < GBK; ++k) {
-            float a[4], b[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                a[i] = As[k][ty * 4 + i];
-                b[i] = Ws[k][tx * 4 + i];
-            }
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-#pragma unroll
-                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
-        }
-        __syncthreads();
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int t = m0 + ty * 4 + i;
-        if (t >= T) continue;
-#pragma unroll
-        for (int j = 0; j < 4; j += 2) {
-            const int c = n0 + tx * 4 + j;
-            if (c < N) epi.pair(t, c, acc[i][j], acc[i][j + 1]);
-        }
-    }
-}
 
 // ------------------------------------------------------------ attention -----
 // O[t][head] = softmax over keys 0..P+t of (Q[t][head] . K) / sqrt(d), times V.
 // One warp per (token, query head); keys read through the page table.
 template <int D>
 __global__ void __launch_bounds__(128) attn_prefill_kernel(const float *Q, const uint16_t *kv,
-                                                           const int *pages, float *O, int P, int T,
-                                                           int nq, int nkv, size_t page_elems,
+                                                           const int *pages, uint16_t *Ohi, uint16_t *Olo,
+                                                           int P, int T, int nq, int nkv, size_t page_elems,
                                                            float qscale) {
     constexpr int EPL = D / 32;
     const int t = blockIdx.x;
@@ -183,7 +147,8 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(const float *Q, const
     }
     const float inv = 1.0f / l;
 #pragma unroll
-    for (int e = 0; e < EPL; ++e) O[(size_t)t * qdim + head * D + lane * EPL + e] = acc[e] * inv;
+    for (int e = 0; e < EPL; ++e)
+        split_store(Ohi, Olo, (size_t)t * qdim + head * D + lane * EPL + e, acc[e] * inv);
 }
 
 // --------------------------------------------------------------- RoPE table --
@@ -199,52 +164,121 @@ __global__ void rope_table_kernel(float2 *rope, int n_pos, int half, double thet
 
 // ================================================================ host =======
 
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        cudaDriverEntryPointQueryResult q;
+        void *p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (EncodeTiledFn)p;
+    }
+    return fn;
+}
+
+// 2-D map over a row-major bf16 matrix [rows][K]; boxes of 64 x box_rows, 128 B swizzle
+static bool encode_2d(CUtensorMap *m, const void *ptr, int rows, int K, int box_rows) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+    cuuint32_t box[2] = {(cuuint32_t)TC_BK, (cuuint32_t)box_rows};
+    cuuint32_t es[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
+    const int T = p.max_chunk;
+    bool ok = encode_2d(&m->ahi, b.Ahi, T, p.H, TC_BM) && encode_2d(&m->alo, b.Alo, T, p.H, TC_BM) &&
+              encode_2d(&m->ohi, b.Ohi, T, p.qdim, TC_BM) && encode_2d(&m->olo, b.Olo, T, p.qdim, TC_BM) &&
+              encode_2d(&m->mhi, b.Mhi, T, p.F, TC_BM) && encode_2d(&m->mlo, b.Mlo, T, p.F, TC_BM);
+    if (!ok) return "cuTensorMapEncodeTiled failed for an activation operand";
+    m->wqkv.resize(p.L);
+    m->wo.resize(p.L);
+    m->wgu.resize(p.L);
+    m->wd.resize(p.L);
+    for (int l = 0; l < p.L; ++l) {
+        const LayerOffsets &lo = p.layer[l];
+        ok = encode_2d(&m->wqkv[l], b.W + lo.wqkv, p.nqkv, p.H, TC_BN) &&
+             encode_2d(&m->wo[l], b.W + lo.wo, p.H, p.qdim, TC_BN) &&
+             encode_2d(&m->wgu[l], b.W + lo.wgu, 2 * p.F, p.H, TC_BN) &&
+             encode_2d(&m->wd[l], b.W + lo.wd, p.H, p.F, TC_BN);
+        if (!ok) return "cuTensorMapEncodeTiled failed for a weight matrix";
+    }
+    static bool attrs = false;
+    if (!attrs) {
+        if (cudaFuncSetAttribute(gemm_tc_kernel<PEpiQKV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)TC_SMEM) != cudaSuccess ||
+            cudaFuncSetAttribute(gemm_tc_kernel<PEpiResidual>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)TC_SMEM) != cudaSuccess ||
+            cudaFuncSetAttribute(gemm_tc_kernel<PEpiSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)TC_SMEM) != cudaSuccess)
+            return "cannot raise the shared-memory limit of the tensor-core GEMM";
+        attrs = true;
+    }
+    return nullptr;
+}
+
 template <class Epi>
-static cudaError_t gemm(const float *A, const uint16_t *W, int T, int N, int K, const Epi &epi,
-                        cudaStream_t st, LaunchHook *hook, const char *name) {
+static cudaError_t gemm(const CUtensorMap &ahi, const CUtensorMap &alo, const CUtensorMap &w, int T, int N, int K,
+                        int *err, const Epi &epi, cudaStream_t st, LaunchHook *hook, const char *name) {
     if (hook) hook->before(name);
-    dim3 grid((N + GBN - 1) / GBN, (T + GBM - 1) / GBM);
-    gemm_simt_kernel<Epi><<<grid, 256, 0, st>>>(A, W, T, N, K, epi);
+    dim3 grid((N + TC_BN - 1) / TC_BN, (T + TC_BM - 1) / TC_BM);
+    gemm_tc_kernel<Epi><<<grid, TC_THREADS, TC_SMEM, st>>>(ahi, alo, w, T, N, K, err, epi);
     if (hook) hook->after(name);
     return cudaGetLastError();
 }
 
-cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, cudaStream_t st, int P, int T,
-                                  int lm_pos_add, LaunchHook *hook) {
+cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMaps &mp, cudaStream_t st, int P,
+                                  int T, int lm_pos_add, LaunchHook *hook) {
     cudaError_t e;
+    int *err = b.ctrl + CTRL_ERR;
     const float qscale = 1.4426950408889634f / sqrtf((float)p.d);
     embed_rows_kernel<<<T, 256, 0, st>>>(b.W + p.w_embed, b.tok, b.X, p.H);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     for (int l = 0; l < p.L; ++l) {
         const LayerOffsets &lo = p.layer[l];
         uint16_t *kvl = b.KV + (size_t)l * p.kv_layer_elems;
-        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.attn_norm, b.A, p.H, p.cfg.rms_eps);
+        // A3 + A4: RMSNorm, QKV (+bias), RoPE, paged KV append
+        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.attn_norm, b.Ahi, b.Alo, p.H, p.cfg.rms_eps);
         PEpiQKV eq = {b.Q, kvl, b.pages, b.rope, p.cfg.qkv_bias ? b.W + lo.bqkv : nullptr, P, p.qdim,
                       p.kvdim, p.d, p.nkv, p.kv_page_elems};
-        if ((e = gemm(b.A, b.W + lo.wqkv, T, p.nqkv, p.H, eq, st, hook, "prefill_qkv")) != cudaSuccess)
+        if ((e = gemm(mp.ahi, mp.alo, mp.wqkv[l], T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
             return e;
+        // A5: causal attention over the cache (earlier chunks + this one)
         dim3 ag(T, (p.nq + 3) / 4);
         if (hook) hook->before("prefill_attention");
         if (p.d == 128)
-            attn_prefill_kernel<128><<<ag, 128, 0, st>>>(b.Q, kvl, b.pages, b.O, P, T, p.nq, p.nkv,
+            attn_prefill_kernel<128><<<ag, 128, 0, st>>>(b.Q, kvl, b.pages, b.Ohi, b.Olo, P, T, p.nq, p.nkv,
                                                         p.kv_page_elems, qscale);
         else
-            attn_prefill_kernel<64><<<ag, 128, 0, st>>>(b.Q, kvl, b.pages, b.O, P, T, p.nq, p.nkv,
+            attn_prefill_kernel<64><<<ag, 128, 0, st>>>(b.Q, kvl, b.pages, b.Ohi, b.Olo, P, T, p.nq, p.nkv,
                                                        p.kv_page_elems, qscale);
         if (hook) hook->after("prefill_attention");
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
-        if ((e = gemm(b.O, b.W + lo.wo, T, p.H, p.qdim, PEpiResidual{b.X, p.H}, st, hook,
+        // A6: O projection + residual
+        if ((e = gemm(mp.ohi, mp.olo, mp.wo[l], T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_o_proj")) != cudaSuccess)
             return e;
-        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.ffn_norm, b.A, p.H, p.cfg.rms_eps);
-        if ((e = gemm(b.A, b.W + lo.wgu, T, 2 * p.F, p.H, PEpiSwiGLU{b.M, p.F}, st, hook,
+        // A7: RMSNorm + gate/up + SwiGLU
+        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.ffn_norm, b.Ahi, b.Alo, p.H, p.cfg.rms_eps);
+        if ((e = gemm(mp.ahi, mp.alo, mp.wgu[l], T, 2 * p.F, p.H, err, PEpiSwiGLU{b.Mhi, b.Mlo, p.F}, st, hook,
                       "prefill_gate_up")) != cudaSuccess)
             return e;
-        if ((e = gemm(b.M, b.W + lo.wd, T, p.H, p.F, PEpiResidual{b.X, p.H}, st, hook,
+        // A8: down projection + residual
+        if ((e = gemm(mp.mhi, mp.mlo, mp.wd[l], T, p.H, p.F, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_down")) != cudaSuccess)
             return e;
     }
     if (lm_pos_add > 0) {
+        // A9 on the chunk's last row only
         if ((e = cudaMemcpyAsync(b.x, b.X + (size_t)(T - 1) * p.H, (size_t)p.H * sizeof(float),
                                  cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
             return e;

@@ -12,9 +12,15 @@ namespace wici {
 
 constexpr int kPage = 16;          // tokens per KV page
 constexpr int kGemvThreads = 288;  // 8 consumer warps + 1 producer warp
-constexpr int kGemvStages = 3;     // ring depth
-constexpr uint32_t kGemvStageMax = 32768;  // bytes per stage (one row of K <= 16384)
-constexpr int kGemvMaxRows = 64;   // rows per stage (bounded by the reduction scratch)
+#ifndef WICI_GEMV_RING_BYTES
+#define WICI_GEMV_RING_BYTES 98304
+#endif
+#ifndef WICI_GEMV_CTAS_PER_SM
+#define WICI_GEMV_CTAS_PER_SM 1
+#endif
+constexpr uint32_t kGemvRingBytes = WICI_GEMV_RING_BYTES;   // shared-memory ring per CTA
+constexpr int kGemvCtasPerSm = WICI_GEMV_CTAS_PER_SM;       // GEMV grid = SMs x this
+constexpr uint32_t kGemvStageMax = 32768;  // one unit (<= 2 rows of hidden <= 8192, or a row of K <= 16384)
 
 struct LayerOffsets {       // bf16 element offsets into the weight arena
     size_t attn_norm, wqkv, bqkv, wo, ffn_norm, wgu, wd;
@@ -32,10 +38,10 @@ struct Plan {
     size_t kv_layer_elems;  // max_pages pages
     size_t kv_elems;
     // workspace (byte offsets)
-    size_t ws_ctrl, ws_hist, ws_x, ws_q, ws_o, ws_m, ws_logits, ws_amax, ws_attn, ws_rope,
-        ws_pages, ws_tok, ws_X, ws_A, ws_Q, ws_O, ws_M;
+    size_t ws_ctrl, ws_hist, ws_x, ws_q, ws_o, ws_m, ws_logits, ws_amax, ws_rope,
+        ws_pages, ws_tok, ws_X, ws_Q, ws_Ahi, ws_Alo, ws_Ohi,
+        ws_Olo, ws_Mhi, ws_Mlo;
     size_t ws_bytes;
-    int attn_splits;        // flash-decode splits per KV head
     int num_sms;
 };
 

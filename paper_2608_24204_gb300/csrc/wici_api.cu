@@ -27,6 +27,7 @@ struct wici_ctx {
     std::vector<char> loaded;        // per canonical tensor
     int n_required = 0, n_loaded = 0;
     cudaGraphExec_t step_exec = nullptr;
+    PrefillMaps maps;
     int32_t *pinned = nullptr;       // host staging: [0] token in, [1] token out, [2] err
     std::string err;
 };
@@ -109,8 +110,6 @@ const char *wici::make_plan(const wici_config *cfg, int num_sms, Plan *p) {
     P.kv_layer_elems = P.kv_page_elems * P.max_pages;
     P.kv_elems = P.kv_layer_elems * P.L;
 
-    P.attn_splits = (2 * P.num_sms + P.nkv - 1) / P.nkv;
-    if (P.attn_splits < 1) P.attn_splits = 1;
 
     size_t w = 0;
     auto ws = [&](size_t bytes) { size_t o = w; w = align_up(w + bytes, 256); return o; };
@@ -123,15 +122,17 @@ const char *wici::make_plan(const wici_config *cfg, int num_sms, Plan *p) {
     P.ws_m = ws(F * 4);
     P.ws_logits = ws(V * 4);
     P.ws_amax = ws((size_t)P.num_sms * sizeof(int2));
-    P.ws_attn = ws((size_t)P.nkv * P.attn_splits * P.group * (P.d + 2) * 4);
     P.ws_rope = ws((size_t)c.max_tokens * (P.d / 2) * sizeof(float2));
     P.ws_pages = ws((size_t)P.max_pages * 4);
     P.ws_tok = ws(T * 4);
     P.ws_X = ws(T * H * 4);
-    P.ws_A = ws(T * H * 4);
     P.ws_Q = ws(T * P.qdim * 4);
-    P.ws_O = ws(T * P.qdim * 4);
-    P.ws_M = ws(T * F * 4);
+    P.ws_Ahi = ws(T * H * 2);
+    P.ws_Alo = ws(T * H * 2);
+    P.ws_Ohi = ws(T * P.qdim * 2);
+    P.ws_Olo = ws(T * P.qdim * 2);
+    P.ws_Mhi = ws(T * F * 2);
+    P.ws_Mlo = ws(T * F * 2);
     P.ws_bytes = w;
     return nullptr;
 }
@@ -149,15 +150,17 @@ static Bufs make_bufs(const Plan &p, void *W, void *KV, void *WS) {
     b.m = (float *)(ws + p.ws_m);
     b.logits = (float *)(ws + p.ws_logits);
     b.amax = (int2 *)(ws + p.ws_amax);
-    b.attn = (float *)(ws + p.ws_attn);
     b.rope = (float2 *)(ws + p.ws_rope);
     b.pages = (int *)(ws + p.ws_pages);
     b.tok = (int *)(ws + p.ws_tok);
     b.X = (float *)(ws + p.ws_X);
-    b.A = (float *)(ws + p.ws_A);
     b.Q = (float *)(ws + p.ws_Q);
-    b.O = (float *)(ws + p.ws_O);
-    b.M = (float *)(ws + p.ws_M);
+    b.Ahi = (uint16_t *)(ws + p.ws_Ahi);
+    b.Alo = (uint16_t *)(ws + p.ws_Alo);
+    b.Ohi = (uint16_t *)(ws + p.ws_Ohi);
+    b.Olo = (uint16_t *)(ws + p.ws_Olo);
+    b.Mhi = (uint16_t *)(ws + p.ws_Mhi);
+    b.Mlo = (uint16_t *)(ws + p.ws_Mlo);
     return b;
 }
 
@@ -284,6 +287,11 @@ int wici_create(const wici_config *cfg, void *cuda_stream, void *weight_dev, voi
                                  c->stream)) != cudaSuccess)
             break;
         if ((e = enqueue_rope_table(p, c->bufs, c->stream)) != cudaSuccess) break;
+        if (const char *m = make_prefill_maps(p, c->bufs, &c->maps)) {
+            int rc2 = fail(nullptr, WICI_E_CUDA, "create: %s", m);
+            wici_destroy(c);
+            return rc2;
+        }
         e = cudaStreamSynchronize(c->stream);
     } while (0);
     if (e != cudaSuccess) {
@@ -401,7 +409,7 @@ int wici_prefill(wici_ctx *c, const int32_t *tokens, int32_t n, float *logits_ou
         const int T = n - off < p.max_chunk ? n - off : p.max_chunk;
         CUDA_TRY(c, cudaMemcpyAsync(c->bufs.tok, tokens + off, (size_t)T * 4, cudaMemcpyHostToDevice, c->stream));
         const bool last = off + T == n;
-        CUDA_TRY(c, enqueue_prefill_chunk(p, c->bufs, c->stream, c->kv_len + off, T, last ? n : 0, nullptr));
+        CUDA_TRY(c, enqueue_prefill_chunk(p, c->bufs, c->maps, c->stream, c->kv_len + off, T, last ? n : 0, nullptr));
         if (!last) CUDA_TRY(c, cudaStreamSynchronize(c->stream));  // tok buffer is reused by the next chunk
     }
     if (logits_out)
