@@ -148,6 +148,39 @@ int wici_profile_decode(wici_ctx *ctx, int32_t n_steps, const char **names, int3
  * WICI_E_TIMEOUT when the wait gave up as designed (the expected result). */
 int wici_check_bounded_wait(void *cuda_stream, int64_t limit_ns);
 
+/* Final RMSNorm + LM head + greedy argmax of one hidden vector, for callers
+ * that cannot allocate device memory.  The paper has no counterpart: WiCi's
+ * GPU work runs inside the application's own allocations.
+ *
+ * Who needs it: a caller whose device memory is owned by someone else, e.g.
+ * an engine or framework that hands out every byte from its own pool and
+ * forbids side allocations, or a latency-critical thread where cudaMalloc's
+ * possible implicit synchronisation or failure cannot be afforded.  Such a
+ * caller can still pass its input and output buffers, but cannot give the
+ * kernel scratch space; here the scratch (control words and one argmax
+ * partial per CTA, about 9 KB) is a fixed array compiled into the library,
+ * which every GPU that loads the library keeps until the process exits.
+ *
+ *   lm_head_dev    device bf16 [vocab, hidden], row-major (y = W x)
+ *   norm_gain_dev  device bf16 [hidden], final RMSNorm gain
+ *   x_dev          device fp32 [hidden], the hidden vector
+ *   logits_dev     device fp32 [vocab], receives W . RMSNorm(x)
+ *   token_dev      device int32 [1], receives the argmax (lowest index on ties)
+ * All work is enqueued on cuda_stream (a cudaStream_t, NULL for the legacy
+ * stream); the call does not synchronise.  The device is the current one.
+ * Limits: hidden a multiple of 8 in [8, 16384]; vocab >= 1; the current GPU
+ * may have at most 1024 SMs (one scratch partial per CTA); anything else
+ * returns WICI_E_ARG with the reason in wici_last_error(NULL).
+ * The call allocates nothing: no cudaMalloc, no cudaFree, no allocating
+ * library routine.  The first call on a device looks up the scratch array's
+ * device address for that device (make that first call before any stream
+ * capture).  Calls share the one scratch array, which keeps the last call's
+ * contents (the ticket word is cleared at the start of every call), so calls
+ * that can overlap on the GPU race: order them on one stream. */
+int wici_lm_head_argmax_noalloc(void *cuda_stream, const void *lm_head_dev, const void *norm_gain_dev,
+                                const float *x_dev, int32_t hidden, int32_t vocab, float rms_eps,
+                                float *logits_dev, int32_t *token_dev);
+
 /* Destroy the context (frees only what the library allocated). */
 void wici_destroy(wici_ctx *ctx);
 

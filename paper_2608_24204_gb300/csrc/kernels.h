@@ -52,6 +52,13 @@ struct LaunchHook {
 // One-time per-process kernel attributes (dynamic shared memory limits).
 cudaError_t setup_kernels();
 
+// Final RMSNorm + LM head + argmax of a caller-given row x [H] against W [V][H]
+// with caller-given scratch: ctrl (CTRL_WORDS ints, zeroed), partials (grid
+// int2) and hist (>= 1 int).  The token lands in ctrl[CTRL_TOKEN].
+cudaError_t enqueue_lm_head_argmax_raw(const uint16_t *W, const uint16_t *gain, const float *x, int H, int V,
+                                       float eps, float *logits, int *ctrl, int2 *partials, int *hist, int grid,
+                                       cudaStream_t st);
+
 // Whole decode step for the token in ctrl[CTRL_TOKEN] at position ctrl[CTRL_POS]:
 // 5 launches per layer + the LM head.  `pdl` enables programmatic dependent launch.
 cudaError_t enqueue_decode_step(const Plan &p, const Bufs &b, cudaStream_t st, bool pdl,
@@ -67,6 +74,9 @@ cudaError_t enqueue_lm_head(const Plan &p, const Bufs &b, cudaStream_t st, bool 
 // LM head, which advances ctrl[CTRL_POS] by lm_pos_add.
 cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMaps &maps,
                                   cudaStream_t st, int P, int T, int lm_pos_add, LaunchHook *hook);
+
+// Sets the per-thread message returned by wici_last_error(NULL).
+void set_thread_error(const char *msg);
 
 // RoPE table for positions [0, max_tokens).
 cudaError_t enqueue_rope_table(const Plan &p, const Bufs &b, cudaStream_t st);

@@ -745,6 +745,33 @@ cudaError_t enqueue_lm_head(const Plan &p, const Bufs &b, cudaStream_t st, bool 
     return launch_gemv(p, g, e, st, pdl, hook, "lm_head_argmax");
 }
 
+cudaError_t enqueue_lm_head_argmax_raw(const uint16_t *W, const uint16_t *gain, const float *x, int H, int V,
+                                       float eps, float *logits, int *ctrl, int2 *partials, int *hist, int grid,
+                                       cudaStream_t st) {
+    GemvIn g = {};
+    g.W = W;
+    g.K = H;
+    g.n_units = V;
+    g.rpu = 1;
+    g.in = x;
+    g.gain = gain;
+    g.ctrl = ctrl;
+    g.eps = eps;
+    ring_geometry(g);
+    void *fn = gemv_fn<EpiArgmax>(g.K);
+    if (!fn || g.ups < 1) return cudaErrorInvalidValue;
+    EpiArgmax e = {};
+    e.logits = logits;
+    e.partial = partials;
+    e.ctrl = ctrl;
+    e.hist = hist;
+    e.pos_add = 0;
+    e.best = -INFINITY;
+    e.bidx = 0x7fffffff;
+    return launch(reinterpret_cast<void (*)(const GemvIn, const EpiArgmax)>(fn), dim3(grid), dim3(kGemvThreads),
+                  gemv_smem_bytes(g.stages, g.slot_bytes), st, false, g, e);
+}
+
 cudaError_t enqueue_decode_step(const Plan &p, const Bufs &b, cudaStream_t st, bool pdl,
                                 LaunchHook *hook) {
     cudaError_t e;

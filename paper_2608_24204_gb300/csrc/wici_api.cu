@@ -17,6 +17,9 @@ using namespace wici;
 
 static thread_local std::string g_thread_err;
 
+// lets other translation units report an error for wici_last_error(NULL)
+void wici::set_thread_error(const char *msg) { g_thread_err = msg; }
+
 struct wici_ctx {
     Plan plan;
     Bufs bufs;

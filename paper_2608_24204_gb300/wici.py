@@ -22,7 +22,7 @@ STATUS_NAMES = {0: "WICI_OK", -1: "WICI_E_ARG", -2: "WICI_E_STATE", -3: "WICI_E_
 # the entry points declared in include/wici.h
 EXPORTS = ("wici_get_sizes", "wici_create", "wici_load_weights", "wici_prefill", "wici_decode_step",
            "wici_decode", "wici_reset", "wici_set_page_table", "wici_kv_len", "wici_last_error",
-           "wici_profile_decode", "wici_check_bounded_wait", "wici_destroy")
+           "wici_profile_decode", "wici_check_bounded_wait", "wici_destroy", "wici_lm_head_argmax_noalloc")
 
 
 class wici_config(ctypes.Structure):
@@ -71,9 +71,10 @@ def lib():
         L.wici_check_bounded_wait.argtypes = [vp, i64]
         L.wici_destroy.argtypes = [vp]
         L.wici_destroy.restype = None
+        L.wici_lm_head_argmax_noalloc.argtypes = [vp, vp, vp, vp, i32, i32, ctypes.c_float, vp, vp]
         for name in ("wici_get_sizes", "wici_create", "wici_load_weights", "wici_prefill", "wici_decode_step",
                      "wici_decode", "wici_reset", "wici_set_page_table", "wici_profile_decode",
-                     "wici_check_bounded_wait"):
+                     "wici_check_bounded_wait", "wici_lm_head_argmax_noalloc"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -182,6 +183,15 @@ def wici_check_bounded_wait(stream: int, limit_ns: int) -> int:
 
 def wici_destroy(ctx) -> None:
     lib().wici_destroy(ctx)
+
+
+def wici_lm_head_argmax_noalloc(stream: int, lm_head_dev: int, norm_gain_dev: int, x_dev: int, hidden: int,
+                                vocab: int, rms_eps: float, logits_dev: int, token_dev: int) -> None:
+    """Final RMSNorm + LM head + argmax on device pointers, without any device
+    allocation (for callers whose device memory is owned elsewhere); the
+    scratch is a fixed array inside the library.  Enqueued on `stream`."""
+    _check(lib().wici_lm_head_argmax_noalloc(stream, lm_head_dev, norm_gain_dev, x_dev, hidden, vocab, rms_eps,
+                                              logits_dev, token_dev))
 
 
 # ------------------------------------------------------------- convenience
