@@ -398,15 +398,17 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const GemvIn g, c
 }
 
 // ------------------------------------------------------------ flash-decode ----
-// Grid (kFdSplits, nkv) in clusters of kFdSplits CTAs: one cluster per KV head g.
-// Block = 32 * (group + 1) threads: warp w < group is query head g*group+w, the
-// last warp streams this CTA's KV pages (K and V blocks of head g, 16 x d bf16
-// each, contiguous in a page) through a 4-stage TMA ring.  The length comes from
-// the device position, so one captured graph serves every step.  Each query
-// warp keeps an online softmax over its CTA's pages and leaves (m, l, acc[d]) in
-// shared memory; after a cluster barrier the CTA of rank 0 combines the
-// kFdSplits partials over distributed shared memory, in rank order.
-constexpr int kFdStages = 4;
+// Grid (kFdSplits, nkv) in clusters of kFdSplits CTAs: one cluster per KV head g,
+// CTA rank r covering a contiguous range of the cached pages.  Block = group x
+// wph query warps + 1 producer warp.  The producer streams the range's pages (the
+// K and V blocks of head g, 16 x d bf16 each, contiguous in a page) through a
+// kFdStages-slot TMA ring; query warp (j, set) runs an online softmax for query
+// head g*group + j over the pages i = set (mod wph) of the range.  The length
+// comes from the device position, so one captured graph serves every step.  The
+// wph states of a head are merged in shared memory, then the CTA of rank 0
+// combines the kFdSplits CTAs' partials over distributed shared memory, in rank
+// order.
+constexpr int kFdStages = 8;
 constexpr int kFdSplits = 16;   // cluster size (non-portable: 16 > 8)
 
 struct FDArgs {
@@ -415,7 +417,7 @@ struct FDArgs {
     const int *pages;
     int *ctrl;
     float *o;
-    int nkv, group;
+    int nkv, group, wph;
     size_t page_elems;
     float qscale;        // log2(e) / sqrt(d)
 };
@@ -432,23 +434,52 @@ __device__ __forceinline__ void cluster_sync_all() {
 }
 __device__ __forceinline__ uint32_t dsmem_addr(const void *local, uint32_t rank) {
     uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(local)), "r"(rank));
+    asm("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(local)), "r"(rank));
     return r;
 }
-__device__ __forceinline__ float ld_dsmem(uint32_t addr) {
-    float v;
-    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+// plain (reorderable) loads from another CTA's shared memory; ordering against
+// the writes comes from the cluster barrier that precedes them
+__device__ __forceinline__ float2 ld_dsmem2(uint32_t addr) {
+    float2 v;
+    asm("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ float4 ld_dsmem4(uint32_t addr) {
+    float4 v;
+    asm("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
     return v;
 }
 
+// (m, l, acc) online-softmax merge of b into a (log2 domain)
+// An empty state (no keys seen) has m = -inf, l = 0, acc = 0 and is skipped:
+// exp2(m - M) with both maxima -inf would be NaN.
+template <int EPL>
+__device__ __forceinline__ void fd_merge(float &m, float &l, float *acc, float mb, float lb, const float *accb) {
+    if (mb == -INFINITY) return;
+    if (m == -INFINITY) {
+        m = mb;
+        l = lb;
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) acc[e] = accb[e];
+        return;
+    }
+    const float M = fmaxf(m, mb);
+    const float fa = exp2f(m - M), fb = exp2f(mb - M);
+    l = l * fa + lb * fb;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) acc[e] = acc[e] * fa + accb[e] * fb;
+    m = M;
+}
+
 template <int D>
-__global__ void __launch_bounds__(288) flash_decode_kernel(const FDArgs a) {
+__global__ void __launch_bounds__(544, 2) flash_decode_kernel(const FDArgs a) {
     constexpr int EPL = D / 32;
     constexpr uint32_t BLK = kPage * D * 2;     // bytes of one K (or V) block of a page
     extern __shared__ __align__(128) uint8_t fsm[];   // [kFdStages][K block | V block]
     __shared__ __align__(8) uint64_t full_bar[kFdStages], empty_bar[kFdStages];
-    __shared__ __align__(16) float s_part[8][D + 4];  // per query warp: acc[D], m, l
+    __shared__ __align__(16) float s_state[16][D + 4];   // per query warp: acc[D], m, l
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nq = a.group * a.wph;   // query warps
     const int g = blockIdx.y;
     const uint32_t rank = cluster_ctarank();
     int *err = a.ctrl + CTRL_ERR;
@@ -469,93 +500,115 @@ __global__ void __launch_bounds__(288) flash_decode_kernel(const FDArgs a) {
     const int p0 = (int)rank * pps;
     const int n = max(0, min(npages, p0 + pps) - p0);
 
-    if (w == a.group) {  // ---------------------------------------- producer
-        if (lane == 0) {
-            const uint32_t ring0 = smem_u32(fsm);
-            int issued = 0;
-            bool waited = false;
-            for (int i = 0; i < n; ++i) {
-                const int s = i % kFdStages;
-                if (i >= kFdStages &&
-                    !mbar_wait(smem_u32(&empty_bar[s]), ((i / kFdStages) + 1) & 1, err, SITE_FD_EMPTY))
-                    break;
-                // the page holding the current position is written by the preceding kernel
-                if (!waited && p0 + i == npages - 1) {
-                    griddep_wait();
-                    waited = true;
-                }
-                const uint16_t *Kb = a.kv + (size_t)a.pages[p0 + i] * a.page_elems + (size_t)g * kPage * D;
+    if (w == nq) {  // ---------------------------------------------- producer
+        // the whole warp walks the pages so that 32 page-table entries are read at
+        // once (one coalesced load) and handed out by shuffle; lane 0 issues
+        const uint32_t ring0 = smem_u32(fsm);
+        int issued = 0, my_page = 0;
+        bool waited = false;
+        for (int i = 0; i < n; ++i) {
+            if ((i & 31) == 0 && i + lane < n) my_page = a.pages[p0 + i + lane];
+            const int page = __shfl_sync(0xffffffffu, my_page, i & 31);
+            const int s = i % kFdStages;
+            bool ok = true;
+            if (lane == 0 && i >= kFdStages)
+                ok = mbar_wait(smem_u32(&empty_bar[s]), ((i / kFdStages) + 1) & 1, err, SITE_FD_EMPTY);
+            if (!__shfl_sync(0xffffffffu, (int)ok, 0)) break;
+            // the page holding the current position is written by the preceding kernel
+            if (!waited && p0 + i == npages - 1) {
+                griddep_wait();
+                waited = true;
+            }
+            if (lane == 0) {
+                const uint16_t *Kb = a.kv + (size_t)page * a.page_elems + (size_t)g * kPage * D;
                 const uint16_t *Vb = Kb + (size_t)a.nkv * kPage * D;
                 const uint32_t fb = smem_u32(&full_bar[s]);
                 mbar_arrive_expect_tx(fb, 2 * BLK);
                 bulk_g2s(ring0 + s * 2 * BLK, Kb, BLK, fb);
                 bulk_g2s(ring0 + s * 2 * BLK + BLK, Vb, BLK, fb);
-                issued = i + 1;
             }
+            issued = i + 1;
+        }
+        if (lane == 0)
             for (int i = max(0, issued - kFdStages); i < issued; ++i)
                 mbar_wait(smem_u32(&full_bar[i % kFdStages]), (i / kFdStages) & 1, err, SITE_FD_DRAIN);
-        }
         __syncwarp();
     } else {  // ------------------------------------------------- query warps
         griddep_wait();
-        const int head = g * a.group + w;
+        const int j = w % a.group, set = w / a.group;
+        const int head = g * a.group + j;
         float qv[EPL], acc[EPL];
-#pragma unroll
-        for (int e = 0; e < EPL; ++e) {
-            qv[e] = a.q[head * D + lane * EPL + e] * a.qscale;
-            acc[e] = 0.f;
+        if constexpr (EPL == 4) {
+            const float4 q4 = *reinterpret_cast<const float4 *>(a.q + head * D + lane * 4);
+            qv[0] = q4.x * a.qscale; qv[1] = q4.y * a.qscale; qv[2] = q4.z * a.qscale; qv[3] = q4.w * a.qscale;
+        } else {
+            const float2 q2 = *reinterpret_cast<const float2 *>(a.q + head * D + lane * 2);
+            qv[0] = q2.x * a.qscale; qv[1] = q2.y * a.qscale;
         }
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
         float m = -INFINITY, l = 0.f;
+        const int key = lane >> 1;   // the key whose score this lane ends with
         bool ok = true;
-        for (int i = 0; i < n && ok; ++i) {
+        for (int i = set; i < n && ok; i += a.wph) {
             const int s = i % kFdStages;
             ok = mbar_wait(smem_u32(&full_bar[s]), (i / kFdStages) & 1, err, SITE_FD_FULL);
             if (!ok) break;
             const uint8_t *Ks = fsm + (size_t)s * 2 * BLK;
             const uint8_t *Vs = Ks + BLK;
             const int ntok = min(kPage, len - (p0 + i) * kPage);
+            // partial dot products of this lane's d-slice with the 16 keys
             float sc[kPage];
 #pragma unroll
             for (int t = 0; t < kPage; ++t) {
                 const uint8_t *kr = Ks + (t * D + lane * EPL) * 2;
                 if constexpr (EPL == 4) {
                     const uint2 kw = *reinterpret_cast<const uint2 *>(kr);
-                    sc[t] = qv[0] * bf16lo(kw.x) + qv[1] * bf16hi(kw.x) + qv[2] * bf16lo(kw.y) +
-                            qv[3] * bf16hi(kw.y);
+                    sc[t] = qv[0] * bf16lo(kw.x) + qv[1] * bf16hi(kw.x) + qv[2] * bf16lo(kw.y) + qv[3] * bf16hi(kw.y);
                 } else {
                     const uint32_t kw = *reinterpret_cast<const uint32_t *>(kr);
                     sc[t] = qv[0] * bf16lo(kw) + qv[1] * bf16hi(kw);
                 }
             }
+            // transposed butterfly: lanes 2k and 2k+1 end with the full score of key k
 #pragma unroll
-            for (int o = 16; o > 0; o >>= 1)
+            for (int o = 16, cnt = kPage; o > 0; o >>= 1) {
+                if (cnt > 1) {
+                    const bool up = (lane & o) != 0;
 #pragma unroll
-                for (int t = 0; t < kPage; ++t) sc[t] += __shfl_xor_sync(0xffffffffu, sc[t], o);
-            float mx = m;
-#pragma unroll
-            for (int t = 0; t < kPage; ++t) {
-                if (t >= ntok) sc[t] = -INFINITY;
-                mx = fmaxf(mx, sc[t]);
+                    for (int t = 0; t < cnt / 2; ++t) {
+                        const float send = up ? sc[t] : sc[t + cnt / 2];
+                        const float keep = up ? sc[t + cnt / 2] : sc[t];
+                        sc[t] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+                    }
+                    cnt >>= 1;
+                } else {
+                    sc[0] += __shfl_xor_sync(0xffffffffu, sc[0], o);
+                }
             }
+            const float my = key < ntok ? sc[0] : -INFINITY;   // slots past the length are masked
+            const float mx = fmaxf(m, warp_max(my));
             const float corr = exp2f(m - mx);
-            l *= corr;
+            const float pme = exp2f(my - mx);                  // 0 for masked keys
+            l = l * corr + pme;   // per-lane share of the denominator (every key is held by two lanes)
 #pragma unroll
             for (int e = 0; e < EPL; ++e) acc[e] *= corr;
 #pragma unroll
             for (int t = 0; t < kPage; ++t) {
-                // slots past the length are never read: unwritten cache memory may hold NaN bits
-                if (t >= ntok) break;
-                const float pt = exp2f(sc[t] - mx);
-                l += pt;
+                // slots past the length are never used: unwritten cache memory may hold NaN bits
+                const bool valid = t < ntok;
+                const float pt = __shfl_sync(0xffffffffu, pme, 2 * t);
                 const uint8_t *vr = Vs + (t * D + lane * EPL) * 2;
                 if constexpr (EPL == 4) {
-                    const uint2 vw = *reinterpret_cast<const uint2 *>(vr);
+                    uint2 vw = *reinterpret_cast<const uint2 *>(vr);
+                    if (!valid) vw = make_uint2(0u, 0u);
                     acc[0] = fmaf(pt, bf16lo(vw.x), acc[0]);
                     acc[1] = fmaf(pt, bf16hi(vw.x), acc[1]);
                     acc[2] = fmaf(pt, bf16lo(vw.y), acc[2]);
                     acc[3] = fmaf(pt, bf16hi(vw.y), acc[3]);
                 } else {
-                    const uint32_t vw = *reinterpret_cast<const uint32_t *>(vr);
+                    uint32_t vw = *reinterpret_cast<const uint32_t *>(vr);
+                    if (!valid) vw = 0u;
                     acc[0] = fmaf(pt, bf16lo(vw), acc[0]);
                     acc[1] = fmaf(pt, bf16hi(vw), acc[1]);
                 }
@@ -564,37 +617,73 @@ __global__ void __launch_bounds__(288) flash_decode_kernel(const FDArgs a) {
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&empty_bar[s]));
         }
+        l = warp_sum(l) * 0.5f;
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) s_part[w][lane * EPL + e] = acc[e];
+        for (int e = 0; e < EPL; ++e) s_state[w][lane * EPL + e] = acc[e];
         if (lane == 0) {
-            s_part[w][D] = m;
-            s_part[w][D + 1] = l;
+            s_state[w][D] = m;
+            s_state[w][D + 1] = l;
+        }
+        // merge the wph page sets of each head into set 0's slot (fixed set order)
+        asm volatile("bar.sync 1, %0;" ::"r"(32 * nq) : "memory");
+        if (set == 0) {
+            for (int t = 1; t < a.wph; ++t) {
+                const float *o = s_state[t * a.group + j];
+                float ob[EPL];
+#pragma unroll
+                for (int e = 0; e < EPL; ++e) ob[e] = o[lane * EPL + e];
+                fd_merge<EPL>(m, l, acc, o[D], o[D + 1], ob);
+            }
+            // all reads of the other sets' states are done before set 0 overwrites its own
+            __syncwarp();
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) s_state[j][lane * EPL + e] = acc[e];
+            if (lane == 0) {
+                s_state[j][D] = m;
+                s_state[j][D + 1] = l;
+            }
         }
     }
-    cluster_sync_all();   // every CTA's partials are written and visible to the cluster
+    cluster_sync_all();   // every CTA's merged partials are written and visible to the cluster
     if (rank == 0 && w < a.group) {
         const int head = g * a.group + w;
-        float ms = -INFINITY, ls = 0.f;
-        if (lane < kFdSplits) {
-            ms = ld_dsmem(dsmem_addr(&s_part[w][D], lane));
-            ls = ld_dsmem(dsmem_addr(&s_part[w][D + 1], lane));
-        }
-        const float M = warp_max(ms);
-        const float f = lane < kFdSplits ? exp2f(ms - M) : 0.f;   // empty splits: exp2(-inf) = 0
-        const float L = warp_sum(ls * f);
+        // lanes 0..15 read the (m, l) of one split each
+        float2 ml = make_float2(-INFINITY, 0.f);
+        if (lane < kFdSplits) ml = ld_dsmem2(dsmem_addr(&s_state[w][D], lane));
+        const float M = warp_max(ml.x);
+        const float f = lane < kFdSplits ? exp2f(ml.x - M) : 0.f;   // empty splits: exp2(-inf) = 0
+        const float L = warp_sum(ml.y * f);
         float out[EPL];
 #pragma unroll
         for (int e = 0; e < EPL; ++e) out[e] = 0.f;
+        if constexpr (EPL == 4) {
+            float4 v[kFdSplits];
 #pragma unroll
-        for (int s = 0; s < kFdSplits; ++s) {
-            const float fs = __shfl_sync(0xffffffffu, f, s);
-            const uint32_t ra = dsmem_addr(&s_part[w][lane * EPL], (uint32_t)s);
+            for (int s = 0; s < kFdSplits; ++s) v[s] = ld_dsmem4(dsmem_addr(&s_state[w][lane * 4], (uint32_t)s));
 #pragma unroll
-            for (int e = 0; e < EPL; ++e) out[e] = fmaf(ld_dsmem(ra + 4 * e), fs, out[e]);
+            for (int s = 0; s < kFdSplits; ++s) {
+                const float fs = __shfl_sync(0xffffffffu, f, s);
+                out[0] = fmaf(v[s].x, fs, out[0]);
+                out[1] = fmaf(v[s].y, fs, out[1]);
+                out[2] = fmaf(v[s].z, fs, out[2]);
+                out[3] = fmaf(v[s].w, fs, out[3]);
+            }
+            const float inv = 1.0f / L;
+            *reinterpret_cast<float4 *>(a.o + head * D + lane * 4) =
+                make_float4(out[0] * inv, out[1] * inv, out[2] * inv, out[3] * inv);
+        } else {
+            float2 v[kFdSplits];
+#pragma unroll
+            for (int s = 0; s < kFdSplits; ++s) v[s] = ld_dsmem2(dsmem_addr(&s_state[w][lane * 2], (uint32_t)s));
+#pragma unroll
+            for (int s = 0; s < kFdSplits; ++s) {
+                const float fs = __shfl_sync(0xffffffffu, f, s);
+                out[0] = fmaf(v[s].x, fs, out[0]);
+                out[1] = fmaf(v[s].y, fs, out[1]);
+            }
+            const float inv = 1.0f / L;
+            *reinterpret_cast<float2 *>(a.o + head * D + lane * 2) = make_float2(out[0] * inv, out[1] * inv);
         }
-        const float inv = 1.0f / L;
-#pragma unroll
-        for (int e = 0; e < EPL; ++e) a.o[head * D + lane * EPL + e] = out[e] * inv;
     }
     cluster_sync_all();   // keep every CTA's shared memory alive until rank 0 has read it
 }
@@ -628,11 +717,15 @@ static cudaError_t launch(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStr
     return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
+// query warps per head: up to 4, at most 16 query warps per CTA (two CTAs fit an SM,
+// so a 16-CTA cluster needs only 8 SMs of a GPC)
+static int fd_wph(int group) { return group >= 4 ? 16 / group : 4; }
+
 template <int D>
 static cudaError_t launch_fd(const Plan &p, const FDArgs &fa, cudaStream_t st, bool pdl) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(kFdSplits, p.nkv);
-    cfg.blockDim = dim3(32 * (p.group + 1));
+    cfg.blockDim = dim3(32 * (fa.group * fa.wph + 1));
     cfg.dynamicSmemBytes = (size_t)kFdStages * 2 * kPage * D * 2;
     cfg.stream = st;
     cudaLaunchAttribute attr[2];
@@ -685,6 +778,12 @@ cudaError_t setup_kernels() {
         return e;
     if ((e = cudaFuncSetAttribute(flash_decode_kernel<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
         cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(flash_decode_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  kFdStages * 2 * kPage * 128 * 2)) != cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(flash_decode_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  kFdStages * 2 * kPage * 64 * 2)) != cudaSuccess)
         return e;
     if ((e = set_gemv_attrs<EpiResidual>()) != cudaSuccess) return e;
     if ((e = set_gemv_attrs<EpiSwiGLU>()) != cudaSuccess) return e;
@@ -799,7 +898,7 @@ cudaError_t enqueue_decode_step(const Plan &p, const Bufs &b, cudaStream_t st, b
         eq.page_elems = p.kv_page_elems;
         if ((e = launch_gemv(p, g, eq, st, pdl && l > 0, hook, "qkv_rope_kvappend")) != cudaSuccess) return e;
         // A5: attention
-        FDArgs fa = {b.q, kvl, b.pages, b.ctrl, b.o, p.nkv, p.group, p.kv_page_elems, qscale};
+        FDArgs fa = {b.q, kvl, b.pages, b.ctrl, b.o, p.nkv, p.group, fd_wph(p.group), p.kv_page_elems, qscale};
         if (hook) hook->before("flash_decode");
         if (p.d == 128)
             e = launch_fd<128>(p, fa, st, pdl);
