@@ -26,8 +26,8 @@ struct Bufs {
     int *pages;       // logical -> physical KV page                         [max_pages]
     int *tok;         // prefill chunk tokens                                [max_chunk]
     float *X;         // prefill residual stream                             [max_chunk][H]
-    float *Q;         // prefill queries after RoPE                          [max_chunk][qdim]
-    // prefill GEMM operands, each an fp32 activation split as hi + lo (bf16 bits)
+    // prefill tensor-core operands, each an fp32 activation split as hi + lo (bf16 bits)
+    uint16_t *Qhi, *Qlo;  // queries after RoPE                               [max_chunk][qdim]
     uint16_t *Ahi, *Alo;  // RMSNorm output                                   [max_chunk][H]
     uint16_t *Ohi, *Olo;  // attention output                                 [max_chunk][qdim]
     uint16_t *Mhi, *Mlo;  // SwiGLU output                                    [max_chunk][F]
@@ -36,6 +36,8 @@ struct Bufs {
 // TMA descriptors of the prefill GEMM operands (built once per context).
 struct PrefillMaps {
     CUtensorMap ahi, alo, ohi, olo, mhi, mlo;          // activations, 128-row boxes
+    CUtensorMap qhi, qlo;                              // queries: [token][head][d], group x tpt boxes
+    CUtensorMap kv;                                    // the whole KV pool: [page][K|V][kv_head][16][d]
     std::vector<CUtensorMap> wqkv, wo, wgu, wd;        // per layer weights, 256-row boxes
 };
 

@@ -1,13 +1,15 @@
 // Prefill: a chunk of T prompt tokens at positions P..P+T-1 through every
 // layer.  The four linear maps of a layer run on the tcgen05 GEMM (gemm_tc.cuh)
-// with fused epilogues (bias + RoPE + paged KV append, residual add, SwiGLU);
-// the kernels around them produce the GEMM operands as bf16 hi/lo pairs.
+// with fused epilogues (bias + RoPE + paged KV append, residual add, SwiGLU)
+// and the causal attention on the tcgen05 attention kernel (attn_tc.cuh); the
+// kernels around them produce the tensor-core operands as bf16 hi/lo pairs.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
 
 #include "common.cuh"
+#include "attn_tc.cuh"
 #include "gemm_tc.cuh"
 #include "kernels.h"
 
@@ -47,8 +49,8 @@ __global__ void rmsnorm_rows_kernel(const float *X, const uint16_t *g, uint16_t 
 
 // --------------------------------------------------------------- epilogues ----
 // pair(t, c, a, b): GEMM output row t, columns (c, c + 1)
-struct PEpiQKV {  // packed QKV columns -> Q (fp32) and K/V pages (bf16)
-    float *Q;
+struct PEpiQKV {  // packed QKV columns -> Q (bf16 hi/lo) and K/V pages (bf16)
+    uint16_t *Qhi, *Qlo;
     uint16_t *kv;
     const int *pages;
     const float2 *rope;
@@ -69,9 +71,9 @@ struct PEpiQKV {  // packed QKV columns -> Q (fp32) and K/V pages (bf16)
             const float ra = a * cs.x - b * cs.y;
             const float rb = b * cs.x + a * cs.y;
             if (c < qdim) {
-                float *qr = Q + (size_t)t * qdim + hd * d;
-                qr[i] = ra;
-                qr[i + half] = rb;
+                const size_t qo = (size_t)t * qdim + hd * d + i;
+                split_store(Qhi, Qlo, qo, ra);
+                split_store(Qhi, Qlo, qo + half, rb);
             } else {
                 uint16_t *kr = page + ((size_t)(hd - qdim / d) * kPage + slot) * d;
                 kr[i] = f32_to_bf16(ra);
@@ -105,51 +107,6 @@ struct PEpiSwiGLU {  // interleaved (gate, up) columns -> M[t][c/2] = silu(g) * 
         split_store(Mhi, Mlo, (size_t)t * ld + (c >> 1), a / (1.0f + expf(-a)) * b);
     }
 };
-
-// ------------------------------------------------------------ attention -----
-// O[t][head] = softmax over keys 0..P+t of (Q[t][head] . K) / sqrt(d), times V.
-// One warp per (token, query head); keys read through the page table.
-template <int D>
-__global__ void __launch_bounds__(128) attn_prefill_kernel(const float *Q, const uint16_t *kv,
-                                                           const int *pages, uint16_t *Ohi, uint16_t *Olo,
-                                                           int P, int T, int nq, int nkv, size_t page_elems,
-                                                           float qscale) {
-    constexpr int EPL = D / 32;
-    const int t = blockIdx.x;
-    const int head = blockIdx.y * 4 + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
-    if (head >= nq) return;
-    const int g = head / (nq / nkv);
-    const int qdim = nq * D;
-    float qv[EPL], acc[EPL];
-#pragma unroll
-    for (int e = 0; e < EPL; ++e) {
-        qv[e] = Q[(size_t)t * qdim + head * D + lane * EPL + e] * qscale;
-        acc[e] = 0.f;
-    }
-    float m = -INFINITY, l = 0.f;
-    const int nkeys = P + t + 1;
-    for (int s = 0; s < nkeys; ++s) {
-        const uint16_t *pg = kv + (size_t)pages[s / kPage] * page_elems;
-        const uint16_t *kr = pg + ((size_t)g * kPage + (s % kPage)) * D + lane * EPL;
-        const uint16_t *vr = kr + (size_t)nkv * kPage * D;
-        float part = 0.f;
-#pragma unroll
-        for (int e = 0; e < EPL; ++e) part = fmaf(qv[e], bf16_to_f32(kr[e]), part);
-        const float sc = warp_sum(part);
-        const float mx = fmaxf(m, sc);
-        const float corr = exp2f(m - mx);
-        const float pt = exp2f(sc - mx);
-        l = l * corr + pt;
-#pragma unroll
-        for (int e = 0; e < EPL; ++e) acc[e] = fmaf(pt, bf16_to_f32(vr[e]), acc[e] * corr);
-        m = mx;
-    }
-    const float inv = 1.0f / l;
-#pragma unroll
-    for (int e = 0; e < EPL; ++e)
-        split_store(Ohi, Olo, (size_t)t * qdim + head * D + lane * EPL + e, acc[e] * inv);
-}
 
 // --------------------------------------------------------------- RoPE table --
 __global__ void rope_table_kernel(float2 *rope, int n_pos, int half, double theta) {
@@ -194,12 +151,44 @@ static bool encode_2d(CUtensorMap *m, const void *ptr, int rows, int K, int box_
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// queries [token][head][d] bf16: boxes of 64 d x `group` heads x tpt tokens (128-byte rows)
+static bool encode_q(CUtensorMap *m, const void *ptr, const Plan &p, int tpt) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)p.d, (cuuint64_t)p.nq, (cuuint64_t)p.max_chunk};
+    cuuint64_t strides[2] = {(cuuint64_t)p.d * 2, (cuuint64_t)p.qdim * 2};
+    cuuint32_t box[3] = {64, (cuuint32_t)p.group, (cuuint32_t)tpt};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// the KV pool of every layer as [page (layer-major)][K|V][kv head][16 slots][d]:
+// boxes of 64 d x 16 slots of one (page, K|V, head)
+static bool encode_kv(CUtensorMap *m, const void *ptr, const Plan &p) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[5] = {(cuuint64_t)p.d, (cuuint64_t)kPage, (cuuint64_t)p.nkv, 2,
+                          (cuuint64_t)p.L * (cuuint64_t)p.max_pages};
+    cuuint64_t strides[4] = {(cuuint64_t)p.d * 2, (cuuint64_t)kPage * p.d * 2, (cuuint64_t)p.nkv * kPage * p.d * 2,
+                             (cuuint64_t)2 * p.nkv * kPage * p.d * 2};
+    cuuint32_t box[5] = {64, (cuuint32_t)kPage, 1, 1, 1};
+    cuuint32_t es[5] = {1, 1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(ptr), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
     const int T = p.max_chunk;
     bool ok = encode_2d(&m->ahi, b.Ahi, T, p.H, TC_BM) && encode_2d(&m->alo, b.Alo, T, p.H, TC_BM) &&
               encode_2d(&m->ohi, b.Ohi, T, p.qdim, TC_BM) && encode_2d(&m->olo, b.Olo, T, p.qdim, TC_BM) &&
               encode_2d(&m->mhi, b.Mhi, T, p.F, TC_BM) && encode_2d(&m->mlo, b.Mlo, T, p.F, TC_BM);
     if (!ok) return "cuTensorMapEncodeTiled failed for an activation operand";
+    const int tpt = attn_tokens_per_tile(p.group);
+    ok = encode_q(&m->qhi, b.Qhi, p, tpt) && encode_q(&m->qlo, b.Qlo, p, tpt) && encode_kv(&m->kv, b.KV, p);
+    if (!ok) return "cuTensorMapEncodeTiled failed for the attention operands";
     m->wqkv.resize(p.L);
     m->wo.resize(p.L);
     m->wgu.resize(p.L);
@@ -219,11 +208,39 @@ const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
             cudaFuncSetAttribute(gemm_tc_kernel<PEpiResidual>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)TC_SMEM) != cudaSuccess ||
             cudaFuncSetAttribute(gemm_tc_kernel<PEpiSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)TC_SMEM) != cudaSuccess)
+                                 (int)TC_SMEM) != cudaSuccess ||
+            cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)(AttnSmem<128>::TOTAL + 1024)) != cudaSuccess ||
+            cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)(AttnSmem<64>::TOTAL + 1024)) != cudaSuccess)
             return "cannot raise the shared-memory limit of the tensor-core GEMM";
         attrs = true;
     }
     return nullptr;
+}
+
+// causal GQA attention of chunk rows [0, T) at positions P.. on the tensor cores
+cudaError_t launch_attn_tc(const Plan &p, const Bufs &b, const PrefillMaps &mp, int layer, int P, int T,
+                           cudaStream_t st) {
+    AttnArgs a;
+    a.Ohi = b.Ohi;
+    a.Olo = b.Olo;
+    a.pages = b.pages;
+    a.err = b.ctrl + CTRL_ERR;
+    a.P = P;
+    a.T = T;
+    a.nq = p.nq;
+    a.group = p.group;
+    a.tpt = attn_tokens_per_tile(p.group);
+    a.layer = layer;
+    a.max_pages = p.max_pages;
+    a.scale_log2 = 1.4426950408889634f / sqrtf((float)p.d);
+    dim3 grid((T + a.tpt - 1) / a.tpt, p.nkv);
+    if (p.d == 128)
+        attn_tc_kernel<128><<<grid, AT_THREADS, AttnSmem<128>::TOTAL + 1024, st>>>(mp.qhi, mp.qlo, mp.kv, a);
+    else
+        attn_tc_kernel<64><<<grid, AT_THREADS, AttnSmem<64>::TOTAL + 1024, st>>>(mp.qhi, mp.qlo, mp.kv, a);
+    return cudaGetLastError();
 }
 
 template <class Epi>
@@ -240,7 +257,6 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
                                   int T, int lm_pos_add, LaunchHook *hook) {
     cudaError_t e;
     int *err = b.ctrl + CTRL_ERR;
-    const float qscale = 1.4426950408889634f / sqrtf((float)p.d);
     embed_rows_kernel<<<T, 256, 0, st>>>(b.W + p.w_embed, b.tok, b.X, p.H);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     for (int l = 0; l < p.L; ++l) {
@@ -248,21 +264,15 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         uint16_t *kvl = b.KV + (size_t)l * p.kv_layer_elems;
         // A3 + A4: RMSNorm, QKV (+bias), RoPE, paged KV append
         rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.attn_norm, b.Ahi, b.Alo, p.H, p.cfg.rms_eps);
-        PEpiQKV eq = {b.Q, kvl, b.pages, b.rope, p.cfg.qkv_bias ? b.W + lo.bqkv : nullptr, P, p.qdim,
+        PEpiQKV eq = {b.Qhi, b.Qlo, kvl, b.pages, b.rope, p.cfg.qkv_bias ? b.W + lo.bqkv : nullptr, P, p.qdim,
                       p.kvdim, p.d, p.nkv, p.kv_page_elems};
         if ((e = gemm(mp.ahi, mp.alo, mp.wqkv[l], T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
             return e;
-        // A5: causal attention over the cache (earlier chunks + this one)
-        dim3 ag(T, (p.nq + 3) / 4);
+        // A5: causal attention over the cache (earlier chunks + this one), tensor cores
         if (hook) hook->before("prefill_attention");
-        if (p.d == 128)
-            attn_prefill_kernel<128><<<ag, 128, 0, st>>>(b.Q, kvl, b.pages, b.Ohi, b.Olo, P, T, p.nq, p.nkv,
-                                                        p.kv_page_elems, qscale);
-        else
-            attn_prefill_kernel<64><<<ag, 128, 0, st>>>(b.Q, kvl, b.pages, b.Ohi, b.Olo, P, T, p.nq, p.nkv,
-                                                       p.kv_page_elems, qscale);
+        e = launch_attn_tc(p, b, mp, l, P, T, st);
         if (hook) hook->after("prefill_attention");
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if (e != cudaSuccess) return e;
         // A6: O projection + residual
         if ((e = gemm(mp.ohi, mp.olo, mp.wo[l], T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_o_proj")) != cudaSuccess)

@@ -39,7 +39,7 @@ struct Plan {
     size_t kv_elems;
     // workspace (byte offsets)
     size_t ws_ctrl, ws_hist, ws_x, ws_q, ws_o, ws_m, ws_logits, ws_amax, ws_rope,
-        ws_pages, ws_tok, ws_X, ws_Q, ws_Ahi, ws_Alo, ws_Ohi,
+        ws_pages, ws_tok, ws_X, ws_Qhi, ws_Qlo, ws_Ahi, ws_Alo, ws_Ohi,
         ws_Olo, ws_Mhi, ws_Mlo;
     size_t ws_bytes;
     int num_sms;

@@ -129,7 +129,8 @@ const char *wici::make_plan(const wici_config *cfg, int num_sms, Plan *p) {
     P.ws_pages = ws((size_t)P.max_pages * 4);
     P.ws_tok = ws(T * 4);
     P.ws_X = ws(T * H * 4);
-    P.ws_Q = ws(T * P.qdim * 4);
+    P.ws_Qhi = ws(T * P.qdim * 2);
+    P.ws_Qlo = ws(T * P.qdim * 2);
     P.ws_Ahi = ws(T * H * 2);
     P.ws_Alo = ws(T * H * 2);
     P.ws_Ohi = ws(T * P.qdim * 2);
@@ -157,7 +158,8 @@ static Bufs make_bufs(const Plan &p, void *W, void *KV, void *WS) {
     b.pages = (int *)(ws + p.ws_pages);
     b.tok = (int *)(ws + p.ws_tok);
     b.X = (float *)(ws + p.ws_X);
-    b.Q = (float *)(ws + p.ws_Q);
+    b.Qhi = (uint16_t *)(ws + p.ws_Qhi);
+    b.Qlo = (uint16_t *)(ws + p.ws_Qlo);
     b.Ahi = (uint16_t *)(ws + p.ws_Ahi);
     b.Alo = (uint16_t *)(ws + p.ws_Alo);
     b.Ohi = (uint16_t *)(ws + p.ws_Ohi);
@@ -284,6 +286,9 @@ int wici_create(const wici_config *cfg, void *cuda_stream, void *weight_dev, voi
         if ((e = setup_kernels()) != cudaSuccess) break;
         if ((e = cudaHostAlloc((void **)&c->pinned, 64, cudaHostAllocDefault)) != cudaSuccess) break;
         if ((e = cudaMemsetAsync(c->bufs.ctrl, 0, CTRL_WORDS * sizeof(int), c->stream)) != cudaSuccess) break;
+        // cache slots past the length are read (and weighted by zero) by the
+        // tensor-core attention: they must hold finite values from the start
+        if ((e = cudaMemsetAsync(c->bufs.KV, 0, p.kv_elems * 2, c->stream)) != cudaSuccess) break;
         std::vector<int> pages(p.max_pages);
         for (int i = 0; i < p.max_pages; ++i) pages[i] = i;
         if ((e = cudaMemcpyAsync(c->bufs.pages, pages.data(), pages.size() * 4, cudaMemcpyHostToDevice,
