@@ -52,6 +52,42 @@ def peaks():
                 "source": "fallback"}
 
 
+KERNEL_SOURCES = ["paper_2608_24204_gb300/csrc/kernels_decode.cu", "paper_2608_24204_gb300/csrc/common.cuh",
+                  "paper_2608_24204_gb300/csrc/plan.h"]
+
+
+def decode_source_hash() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def profiled_traffic(profile: str):
+    """DRAM bytes per launch recorded in a committed ncu summary, or None when the
+    summary is missing or the decode kernel sources changed since the capture."""
+    path = os.path.join(ROOT, "profiles", profile)
+    try:
+        with open(path) as f:
+            text = f.read()
+    except OSError:
+        return None
+    fields = {}
+    for line in text.splitlines():
+        line = line.strip().lstrip("-").strip()
+        if ":" in line:
+            k, v = line.split(":", 1)
+            fields[k.strip()] = v.strip().strip("`")
+    if fields.get("source_sha256") != decode_source_hash():
+        return None
+    try:
+        return int(fields["traffic_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
 class ClockSampler:
     """nvidia-smi clock/throttle samples every 200 ms while running."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -248,7 +284,8 @@ def run_ours(args):
     n_gu, ms_gu = prof["gate_up_swiglu"]
     gu_gbs = gu_bytes / (ms_gu / n_gu / 1000.0) / 1e9
     roofline = {"bound": "hbm", "kernel": "gate_up_swiglu", "achieved": gu_gbs, "peak": pk["hbm_gbs"],
-                "unit": "GB/s", "frac": gu_gbs / pk["hbm_gbs"], "traffic": None,
+                "unit": "GB/s", "frac": gu_gbs / pk["hbm_gbs"],
+                "traffic": profiled_traffic("decode_gemv_gate_up_swiglu_llama3-8b.md"),
                 "peak_source": pk["source"], "bytes_per_launch": gu_bytes,
                 "avg_launch_us": ms_gu / n_gu * 1000.0}
     kernel_share = {k: {"launches": v[0], "ms": v[1]} for k, v in prof.items()}

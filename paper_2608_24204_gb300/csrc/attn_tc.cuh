@@ -5,12 +5,12 @@
 // head g*group + r%group), so each K/V tile serves the whole group.  Keys come
 // from the paged cache in blocks of 64 (four 16-key pages, fetched by 5-D TMA
 // through the page table).  Per block:
-//   S  = (Q_hi + Q_lo) K^T        tcgen05.mma, M=128 rows, N=64 keys, fp32 in TMEM
+//   S  = (Q_0 + Q_1 + Q_2) K^T    tcgen05.mma, M=128 rows, N=64 keys, fp32 in TMEM
 //   softmax (one row per thread, read from TMEM): online max/sum, P = exp2(s - m)
-//   O_blk = (P_hi + P_lo) V       tcgen05.mma, N=d, V read as an MN-major operand
+//   O_blk = (P_0 + P_1 + P_2) V   tcgen05.mma, N=d, V read as an MN-major operand
 //   O = O * corr + O_blk          in registers
-// Q and P are split into two bf16 terms like the GEMM activations; K and V are
-// exact bf16.  Warp roles: 0 TMA producer, 1 TMEM owner + MMA issuer, 2..5
+// Q and P are carried as three bf16 terms like the GEMM activations (fp32
+// precision); K and V are exact bf16.  Warp roles: 0 TMA producer, 1 TMEM owner + MMA issuer, 2..5
 // softmax / output (TMEM lane quadrant = warp % 4).  Every wait is bounded.
 #pragma once
 #include <cuda.h>
@@ -34,13 +34,13 @@ enum : int { SITE_AT_Q = 41, SITE_AT_KVE = 42, SITE_AT_KVF = 43, SITE_AT_S = 44,
 template <int D>
 struct AttnSmem {
     static constexpr int DCH = D / 64;                                   // 64-element d chunks
-    static constexpr uint32_t Q_BYTES = AT_ROWS * D * 2;                 // one of hi / lo
+    static constexpr uint32_t Q_BYTES = AT_ROWS * D * 2;                 // one term
     static constexpr uint32_t KV_BYTES = AT_KEYS * D * 2;                // K (or V) of a block
-    static constexpr uint32_t P_BYTES = AT_ROWS * AT_KEYS * 2;           // one of hi / lo
-    static constexpr uint32_t OFF_QHI = 0, OFF_QLO = Q_BYTES;
-    static constexpr uint32_t OFF_KV = 2 * Q_BYTES;                      // [stage][K | V]
-    static constexpr uint32_t OFF_P = OFF_KV + AT_STAGES * 2 * KV_BYTES; // [hi | lo]
-    static constexpr uint32_t TOTAL = OFF_P + 2 * P_BYTES;
+    static constexpr uint32_t P_BYTES = AT_ROWS * AT_KEYS * 2;           // one term
+    static constexpr uint32_t OFF_Q = 0;                                 // [term]
+    static constexpr uint32_t OFF_KV = kTerms * Q_BYTES;                 // [stage][K | V]
+    static constexpr uint32_t OFF_P = OFF_KV + AT_STAGES * 2 * KV_BYTES; // [term]
+    static constexpr uint32_t TOTAL = OFF_P + kTerms * P_BYTES;
 };
 
 // K-major, 128-byte swizzle, 8-row groups 1024 B apart (Q, K and P operands)
@@ -88,7 +88,7 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 __host__ __device__ constexpr int attn_tokens_per_tile(int group) { return AT_ROWS / group; }
 
 struct AttnArgs {
-    uint16_t *Ohi, *Olo;  // [T][nq * d] outputs (hi / lo)
+    uint16_t *O[kTerms];  // [T][nq * d] output terms
     const int *pages;     // logical -> physical page
     int *err;
     int P, T;             // cached positions before the chunk, chunk length
@@ -99,8 +99,9 @@ struct AttnArgs {
 
 template <int D>
 __global__ void __launch_bounds__(AT_THREADS, 1)
-    attn_tc_kernel(const __grid_constant__ CUtensorMap map_qhi, const __grid_constant__ CUtensorMap map_qlo,
-                   const __grid_constant__ CUtensorMap map_kv, const AttnArgs a) {
+    attn_tc_kernel(const __grid_constant__ CUtensorMap map_q0, const __grid_constant__ CUtensorMap map_q1,
+                   const __grid_constant__ CUtensorMap map_q2, const __grid_constant__ CUtensorMap map_kv,
+                   const AttnArgs a) {
     using L = AttnSmem<D>;
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t q_full, kv_full[AT_STAGES], kv_empty[AT_STAGES], s_full, p_full, o_full;
@@ -144,10 +145,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     if (warp == 0) {
         if (lane == 0) {  // ----------------------------------------------- TMA producer
             const uint32_t qb = smem_u32(&q_full);
-            mbar_arrive_expect_tx(qb, 2u * L::DCH * q_bytes_box);
+            mbar_arrive_expect_tx(qb, (uint32_t)kTerms * L::DCH * q_bytes_box);
             for (int c = 0; c < L::DCH; ++c) {
-                tma_load_3d(base + L::OFF_QHI + c * AT_ROWS * 128, &map_qhi, c * 64, g * a.group, t0, qb);
-                tma_load_3d(base + L::OFF_QLO + c * AT_ROWS * 128, &map_qlo, c * 64, g * a.group, t0, qb);
+                tma_load_3d(base + L::OFF_Q + c * AT_ROWS * 128, &map_q0, c * 64, g * a.group, t0, qb);
+                tma_load_3d(base + L::OFF_Q + L::Q_BYTES + c * AT_ROWS * 128, &map_q1, c * 64, g * a.group, t0, qb);
+                tma_load_3d(base + L::OFF_Q + 2 * L::Q_BYTES + c * AT_ROWS * 128, &map_q2, c * 64, g * a.group, t0,
+                            qb);
             }
             int issued = 0;
             for (int j = 0; j < nb; ++j) {
@@ -189,8 +192,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                     const uint32_t off = (uint32_t)(k / 4) * (AT_ROWS * 128) + 32u * (k % 4);
                     const uint32_t koff = (uint32_t)(k / 4) * (AT_KEYS * 128) + 32u * (k % 4);
                     const uint64_t bd = at_desc_k(kb + koff);
-                    tc_mma(tm_s, at_desc_k(base + L::OFF_QHI + off), bd, idesc_s, k != 0);
-                    tc_mma(tm_s, at_desc_k(base + L::OFF_QLO + off), bd, idesc_s, 1);
+#pragma unroll
+                    for (int t = 0; t < kTerms; ++t)
+                        tc_mma(tm_s, at_desc_k(base + L::OFF_Q + t * L::Q_BYTES + off), bd, idesc_s, (k | t) != 0);
                 }
                 tc_commit(smem_u32(&s_full));
             };
@@ -205,8 +209,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                 for (int k = 0; k < AT_KEYS / 16; ++k) {
                     // 16 keys = two 8-key groups of V rows; P columns 16k..16k+15
                     const uint64_t vd = at_desc_mn(vb + 2048u * k, AT_KEYS * 128);
-                    tc_mma(tm_o, at_desc_k(base + L::OFF_P + 32u * k), vd, idesc_o, k != 0);
-                    tc_mma(tm_o, at_desc_k(base + L::OFF_P + L::P_BYTES + 32u * k), vd, idesc_o, 1);
+#pragma unroll
+                    for (int t = 0; t < kTerms; ++t)
+                        tc_mma(tm_o, at_desc_k(base + L::OFF_P + t * L::P_BYTES + 32u * k), vd, idesc_o, (k | t) != 0);
                 }
                 tc_commit(smem_u32(&o_full));
                 tc_commit(smem_u32(&kv_empty[s]));
@@ -244,25 +249,27 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             const float msafe = mn == -INFINITY ? 0.f : mn;   // rows with nothing visible yet
             const float corr = exp2f(m - msafe);
             float ps = 0.f;
-            // P row r: two bf16 terms, 128-byte swizzled rows (16-byte piece i at i ^ (r % 8))
-            uint8_t *prow_hi = pbase + r * 128;
-            uint8_t *prow_lo = pbase + L::P_BYTES + r * 128;
+            // P row r as three bf16 terms, 128-byte swizzled rows (16-byte piece i at i ^ (r % 8))
+            uint8_t *prow = pbase + r * 128;
 #pragma unroll
             for (int piece = 0; piece < AT_KEYS / 8; ++piece) {
-                uint32_t hw[4], lw[4];
+                uint32_t w0[4], w1[4], w2[4];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     const float p0 = exp2f(sv[piece * 8 + 2 * e] - msafe);
                     const float p1 = exp2f(sv[piece * 8 + 2 * e + 1] - msafe);
                     ps += p0 + p1;
-                    const uint16_t h0 = f32_to_bf16(p0), h1 = f32_to_bf16(p1);
-                    const uint16_t l0 = f32_to_bf16(p0 - bf16_to_f32(h0)), l1 = f32_to_bf16(p1 - bf16_to_f32(h1));
-                    hw[e] = (uint32_t)h0 | ((uint32_t)h1 << 16);
-                    lw[e] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+                    uint16_t a0, a1, a2, b0, b1, b2;
+                    split_bf16x3(p0, a0, a1, a2);
+                    split_bf16x3(p1, b0, b1, b2);
+                    w0[e] = (uint32_t)a0 | ((uint32_t)b0 << 16);
+                    w1[e] = (uint32_t)a1 | ((uint32_t)b1 << 16);
+                    w2[e] = (uint32_t)a2 | ((uint32_t)b2 << 16);
                 }
                 const int sp = (piece ^ (r & 7)) * 16;
-                *reinterpret_cast<uint4 *>(prow_hi + sp) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-                *reinterpret_cast<uint4 *>(prow_lo + sp) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+                *reinterpret_cast<uint4 *>(prow + sp) = make_uint4(w0[0], w0[1], w0[2], w0[3]);
+                *reinterpret_cast<uint4 *>(prow + L::P_BYTES + sp) = make_uint4(w1[0], w1[1], w1[2], w1[3]);
+                *reinterpret_cast<uint4 *>(prow + 2 * L::P_BYTES + sp) = make_uint4(w2[0], w2[1], w2[2], w2[3]);
             }
             l = l * corr + ps;
             m = mn;
@@ -285,17 +292,19 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             const size_t off = (size_t)tok * a.nq * D + (size_t)head * D;
 #pragma unroll
             for (int c = 0; c < D; c += 8) {
-                uint32_t hw[4], lw[4];
+                uint32_t w0[4], w1[4], w2[4];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                    const float v0 = o[c + 2 * e] * inv, v1 = o[c + 2 * e + 1] * inv;
-                    const uint16_t h0 = f32_to_bf16(v0), h1 = f32_to_bf16(v1);
-                    hw[e] = (uint32_t)h0 | ((uint32_t)h1 << 16);
-                    lw[e] = (uint32_t)f32_to_bf16(v0 - bf16_to_f32(h0)) |
-                            ((uint32_t)f32_to_bf16(v1 - bf16_to_f32(h1)) << 16);
+                    uint16_t a0, a1, a2, b0, b1, b2;
+                    split_bf16x3(o[c + 2 * e] * inv, a0, a1, a2);
+                    split_bf16x3(o[c + 2 * e + 1] * inv, b0, b1, b2);
+                    w0[e] = (uint32_t)a0 | ((uint32_t)b0 << 16);
+                    w1[e] = (uint32_t)a1 | ((uint32_t)b1 << 16);
+                    w2[e] = (uint32_t)a2 | ((uint32_t)b2 << 16);
                 }
-                *reinterpret_cast<uint4 *>(a.Ohi + off + c) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-                *reinterpret_cast<uint4 *>(a.Olo + off + c) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+                *reinterpret_cast<uint4 *>(a.O[0] + off + c) = make_uint4(w0[0], w0[1], w0[2], w0[3]);
+                *reinterpret_cast<uint4 *>(a.O[1] + off + c) = make_uint4(w1[0], w1[1], w1[2], w1[3]);
+                *reinterpret_cast<uint4 *>(a.O[2] + off + c) = make_uint4(w2[0], w2[1], w2[2], w2[3]);
             }
         }
     }

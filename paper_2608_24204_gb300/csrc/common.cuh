@@ -38,6 +38,18 @@ __device__ __forceinline__ uint16_t f32_to_bf16(float f) {
     return (uint16_t)(u >> 16);
 }
 
+// Tensor-core operands carry an fp32 activation as kTerms bf16 terms,
+// a = t0 + t1 + t2 with t0 = bf16(a), t1 = bf16(a - t0), t2 = bf16(a - t0 - t1):
+// 24 significant bits, the precision of the fp32 value (bf16x3, one operand).
+constexpr int kTerms = 3;
+
+__device__ __forceinline__ void split_bf16x3(float a, uint16_t &t0, uint16_t &t1, uint16_t &t2) {
+    t0 = f32_to_bf16(a);
+    const float r1 = a - __uint_as_float((uint32_t)t0 << 16);
+    t1 = f32_to_bf16(r1);
+    t2 = f32_to_bf16(r1 - __uint_as_float((uint32_t)t1 << 16));
+}
+
 // ------------------------------------------------------------- mbarriers ----
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return (uint32_t)__cvta_generic_to_shared(p);

@@ -1,19 +1,27 @@
 // Prefill GEMM on the 5th-generation tensor cores (tcgen05 + TMEM + TMA).
 //
-//   C[T][N] = (A_hi + A_lo)[T][K] . W[N][K]^T,  fp32 accumulation in TMEM
+//   C[T][N] = (A_0 + A_1 + A_2)[T][K] . W[N][K]^T,  fp32 accumulation in TMEM
 //
-// A is an fp32 activation split into two bf16 terms (hi = bf16(a),
-// lo = bf16(a - hi)); W is bf16 and exact.  Both products accumulate into one
-// 128x256 fp32 accumulator, giving ~16-bit activation precision on bf16 MMAs
-// (the bf16x2 scheme of Henry, Tang & Heinecke, ARITH 2019, on one operand).
+// A is an fp32 activation carried as kTerms = 3 bf16 terms (split_bf16x3); W is
+// bf16 and exact.  The three products accumulate into one 128x256 fp32
+// accumulator, so the activations keep fp32 precision on bf16 MMAs (the bf16x3
+// scheme of Henry, Tang & Heinecke, ARITH 2019, applied to one operand).
 //
-// One CTA computes one 128x256 output tile with three warp roles:
-//   warp 0      TMA producer: 2-D tiled loads (128-byte swizzle) of A_hi, A_lo
-//               and W k-blocks into a 3-stage shared-memory ring;
+// Accumulation: one tcgen05 accumulator that absorbs the whole K dimension adds
+// each MMA's result with the tensor core's internal alignment, and over K/16
+// k-steps x 3 terms that error grows well past fp32 summation (measured: 4x the
+// logits error of the fp32 CUDA-core path at the Llama-3-8B shape).  So the MMAs
+// accumulate only TC_GROUP k-blocks into one of two TMEM buffers; the epilogue
+// warps fold each finished group into fp32 registers (round-to-nearest adds)
+// while the next group accumulates into the other buffer.
+//
+// One CTA computes one 128x128 output tile with three warp roles:
+//   warp 0      TMA producer: 2-D tiled loads (128-byte swizzle) of the three A
+//               terms and the W k-block into a 3-stage shared-memory ring;
 //   warp 1      allocates 256 TMEM columns and issues tcgen05.mma (one thread);
 //               each stage is released by tcgen05.commit to its "empty" barrier;
-//   warps 2..5  epilogue: tcgen05.ld of their 32 TMEM lanes (one output row per
-//               thread) and the fused epilogue functor on column pairs.
+//   warps 2..5  tcgen05.ld of their 32 TMEM lanes (one output row per thread),
+//               group sums in registers, then the fused epilogue on column pairs.
 // Every mbarrier wait is bounded; a wait that gives up records its site in
 // *err and the CTA still drains its copies, frees TMEM and exits.
 #pragma once
@@ -25,17 +33,18 @@
 
 namespace wici {
 
-constexpr int TC_BM = 128, TC_BN = 256, TC_BK = 64, TC_STAGES = 3, TC_THREADS = 192;
-constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;                 // 16 KB
-constexpr uint32_t TC_B_BYTES = TC_BN * TC_BK * 2;                 // 32 KB
-constexpr uint32_t TC_STAGE_BYTES = 2 * TC_A_BYTES + TC_B_BYTES;   // 64 KB
+constexpr int TC_BM = 128, TC_BN = 128, TC_BK = 64, TC_STAGES = 3, TC_THREADS = 192;
+constexpr int TC_GROUP = 2;                                             // k-blocks per TMEM accumulation
+constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;                      // 16 KB per term
+constexpr uint32_t TC_B_BYTES = TC_BN * TC_BK * 2;                      // 16 KB
+constexpr uint32_t TC_STAGE_BYTES = kTerms * TC_A_BYTES + TC_B_BYTES;   // 64 KB
 constexpr size_t TC_SMEM = (size_t)TC_STAGES * TC_STAGE_BYTES + 1024;
-constexpr uint32_t TC_TMEM_COLS = 256;
+constexpr uint32_t TC_TMEM_COLS = 2 * TC_BN;                            // two accumulator buffers
 
-enum : int { SITE_TC_EMPTY = 21, SITE_TC_FULL = 22, SITE_TC_ACCUM = 23, SITE_TC_DRAIN = 24 };
+enum : int { SITE_TC_EMPTY = 21, SITE_TC_FULL = 22, SITE_TC_ACCUM = 23, SITE_TC_DRAIN = 24, SITE_TC_FREE = 25 };
 
 // instruction descriptor of tcgen05.mma.kind::f16: D fp32, A and B bf16, both
-// K-major, M = 128, N = 256
+// K-major, M = 128, N = TC_BN
 __host__ __device__ constexpr uint32_t tc_idesc() {
     return (1u << 4)                      // D format: f32
            | (1u << 7)                    // A format: bf16
@@ -100,16 +109,19 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, float *v) {
 // Epi::pair(t, c, v0, v1): output row t, columns (c, c + 1)
 template <class Epi>
 __global__ void __launch_bounds__(TC_THREADS, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap map_ahi, const __grid_constant__ CUtensorMap map_alo,
-                   const __grid_constant__ CUtensorMap map_w, int T, int N, int K, int *err, const Epi epi) {
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_a1,
+                   const __grid_constant__ CUtensorMap map_a2, const __grid_constant__ CUtensorMap map_w, int T,
+                   int N, int K, int *err, const Epi epi) {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full_bar[TC_STAGES], empty_bar[TC_STAGES], accum_bar;
+    __shared__ __align__(8) uint64_t full_bar[TC_STAGES], empty_bar[TC_STAGES], acc_full[2], acc_free[2];
     __shared__ uint32_t s_tmem;
     __shared__ int s_issued;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n0 = blockIdx.x * TC_BN, m0 = blockIdx.y * TC_BM;
+    // M tiles vary fastest: the CTAs that run together share one weight tile through L2
+    const int m0 = blockIdx.x * TC_BM, n0 = blockIdx.y * TC_BN;
     const int nk = (K + TC_BK - 1) / TC_BK;
+    const int ngroups = (nk + TC_GROUP - 1) / TC_GROUP;
     const uint32_t base = (smem_u32(smem_raw) + 1023u) & ~1023u;
 
     if (threadIdx.x == 0) {
@@ -117,7 +129,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             mbar_init(smem_u32(&full_bar[s]), 1);
             mbar_init(smem_u32(&empty_bar[s]), 1);
         }
-        mbar_init(smem_u32(&accum_bar), 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&acc_full[b]), 1);
+            mbar_init(smem_u32(&acc_free[b]), 4);
+        }
         fence_barrier_init();
         s_issued = 0;
     }
@@ -143,9 +158,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                 const uint32_t st = base + (uint32_t)s * TC_STAGE_BYTES;
                 const uint32_t fb = smem_u32(&full_bar[s]);
                 mbar_arrive_expect_tx(fb, TC_STAGE_BYTES);
-                tma_load_2d(st, &map_ahi, kb * TC_BK, m0, fb);
-                tma_load_2d(st + TC_A_BYTES, &map_alo, kb * TC_BK, m0, fb);
-                tma_load_2d(st + 2 * TC_A_BYTES, &map_w, kb * TC_BK, n0, fb);
+                tma_load_2d(st, &map_a0, kb * TC_BK, m0, fb);
+                tma_load_2d(st + TC_A_BYTES, &map_a1, kb * TC_BK, m0, fb);
+                tma_load_2d(st + 2 * TC_A_BYTES, &map_a2, kb * TC_BK, m0, fb);
+                tma_load_2d(st + kTerms * TC_A_BYTES, &map_w, kb * TC_BK, n0, fb);
                 issued = kb + 1;
             }
             s_issued = issued;
@@ -154,36 +170,61 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (lane == 0) {  // ------------------------------------------- MMA issuer
             constexpr uint32_t idesc = tc_idesc();
             bool ok = true;
-            for (int kb = 0; kb < nk && ok; ++kb) {
-                const int s = kb % TC_STAGES;
-                ok = mbar_wait(smem_u32(&full_bar[s]), (kb / TC_STAGES) & 1, err, SITE_TC_FULL);
-                if (!ok) break;
+            for (int gi = 0; gi < ngroups && ok; ++gi) {
+                const int b = gi & 1;
+                // the epilogue must have read this buffer's previous group
+                if (gi >= 2 && !(ok = mbar_wait(smem_u32(&acc_free[b]), ((gi / 2) + 1) & 1, err, SITE_TC_FREE)))
+                    break;
                 tc_fence_after();
-                const uint32_t st = base + (uint32_t)s * TC_STAGE_BYTES;
+                const uint32_t acc = tmem + (uint32_t)(b * TC_BN);
+                const int kb1 = min(nk, (gi + 1) * TC_GROUP);
+                for (int kb = gi * TC_GROUP; kb < kb1; ++kb) {
+                    const int s = kb % TC_STAGES;
+                    ok = mbar_wait(smem_u32(&full_bar[s]), (kb / TC_STAGES) & 1, err, SITE_TC_FULL);
+                    if (!ok) break;
+                    tc_fence_after();
+                    const uint32_t st = base + (uint32_t)s * TC_STAGE_BYTES;
 #pragma unroll
-                for (int k = 0; k < TC_BK / 16; ++k) {
-                    const uint64_t bd = tc_desc_sw128(st + 2 * TC_A_BYTES + 32 * k);
-                    tc_mma(tmem, tc_desc_sw128(st + 32 * k), bd, idesc, (kb | k) != 0);
-                    tc_mma(tmem, tc_desc_sw128(st + TC_A_BYTES + 32 * k), bd, idesc, 1);
+                    for (int k = 0; k < TC_BK / 16; ++k) {
+                        const uint64_t bd = tc_desc_sw128(st + kTerms * TC_A_BYTES + 32 * k);
+#pragma unroll
+                        for (int t = 0; t < kTerms; ++t)
+                            tc_mma(acc, tc_desc_sw128(st + t * TC_A_BYTES + 32 * k), bd, idesc,
+                                   (kb != gi * TC_GROUP || k != 0 || t != 0));
+                    }
+                    tc_commit(smem_u32(&empty_bar[s]));
                 }
-                tc_commit(smem_u32(&empty_bar[s]));
+                tc_commit(smem_u32(&acc_full[b]));  // fires when this group's MMAs have completed
             }
-            tc_commit(smem_u32(&accum_bar));  // fires when every MMA issued above has completed
         }
     } else {  // ------------------------------------------------------- epilogue
-        const bool ok = mbar_wait(smem_u32(&accum_bar), 0, err, SITE_TC_ACCUM);
-        tc_fence_after();
         const int q = warp & 3;                 // TMEM lane quadrant of this warp
         const int t = m0 + q * 32 + lane;
-        for (int c0 = 0; c0 < TC_BN; c0 += 32) {
-            float v[32];
-            tc_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, v);
-            if (ok && t < T) {
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        float sum[TC_BN];
 #pragma unroll
-                for (int j = 0; j < 32; j += 2) {
-                    const int c = n0 + c0 + j;
-                    if (c < N) epi.pair(t, c, v[j], v[j + 1]);
-                }
+        for (int c = 0; c < TC_BN; ++c) sum[c] = 0.f;
+        bool ok = true;
+        for (int gi = 0; gi < ngroups && ok; ++gi) {
+            const int b = gi & 1;
+            ok = mbar_wait(smem_u32(&acc_full[b]), (gi / 2) & 1, err, SITE_TC_ACCUM);
+            tc_fence_after();
+#pragma unroll
+            for (int c0 = 0; c0 < TC_BN; c0 += 32) {
+                float v[32];
+                tc_ld32(tmem + lane_base + (uint32_t)(b * TC_BN + c0), v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) sum[c0 + i] += v[i];
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&acc_free[b]));
+        }
+        if (ok && t < T) {
+#pragma unroll
+            for (int j = 0; j < TC_BN; j += 2) {
+                const int c = n0 + j;
+                if (c < N) epi.pair(t, c, sum[j], sum[j + 1]);
             }
         }
     }

@@ -6,6 +6,7 @@
 
 #include <vector>
 
+#include "common.cuh"
 #include "plan.h"
 
 namespace wici {
@@ -26,17 +27,17 @@ struct Bufs {
     int *pages;       // logical -> physical KV page                         [max_pages]
     int *tok;         // prefill chunk tokens                                [max_chunk]
     float *X;         // prefill residual stream                             [max_chunk][H]
-    // prefill tensor-core operands, each an fp32 activation split as hi + lo (bf16 bits)
-    uint16_t *Qhi, *Qlo;  // queries after RoPE                               [max_chunk][qdim]
-    uint16_t *Ahi, *Alo;  // RMSNorm output                                   [max_chunk][H]
-    uint16_t *Ohi, *Olo;  // attention output                                 [max_chunk][qdim]
-    uint16_t *Mhi, *Mlo;  // SwiGLU output                                    [max_chunk][F]
+    // prefill tensor-core operands: each fp32 activation as kTerms bf16 terms
+    uint16_t *Q[kTerms];  // queries after RoPE                               [max_chunk][qdim]
+    uint16_t *A[kTerms];  // RMSNorm output                                   [max_chunk][H]
+    uint16_t *O[kTerms];  // attention output                                 [max_chunk][qdim]
+    uint16_t *M[kTerms];  // SwiGLU output                                    [max_chunk][F]
 };
 
 // TMA descriptors of the prefill GEMM operands (built once per context).
 struct PrefillMaps {
-    CUtensorMap ahi, alo, ohi, olo, mhi, mlo;          // activations, 128-row boxes
-    CUtensorMap qhi, qlo;                              // queries: [token][head][d], group x tpt boxes
+    CUtensorMap a[kTerms], o[kTerms], m[kTerms];       // GEMM activations, 128-row boxes
+    CUtensorMap q[kTerms];                             // queries: [token][head][d], group x tpt boxes
     CUtensorMap kv;                                    // the whole KV pool: [page][K|V][kv_head][16][d]
     std::vector<CUtensorMap> wqkv, wo, wgu, wd;        // per layer weights, 256-row boxes
 };

@@ -15,12 +15,18 @@
 
 namespace wici {
 
-// a = hi + lo with hi = bf16(a), lo = bf16(a - hi)
-__device__ __forceinline__ void split_store(uint16_t *hi, uint16_t *lo, size_t i, float a) {
-    const uint16_t h = f32_to_bf16(a);
-    hi[i] = h;
-    lo[i] = f32_to_bf16(a - bf16_to_f32(h));
+// store a as its three bf16 terms
+__device__ __forceinline__ void split_store(uint16_t *const *t, size_t i, float a) {
+    uint16_t t0, t1, t2;
+    split_bf16x3(a, t0, t1, t2);
+    t[0][i] = t0;
+    t[1][i] = t1;
+    t[2][i] = t2;
 }
+
+struct Terms {   // kTerms pointers passed by value to kernels
+    uint16_t *p[kTerms];
+};
 
 // ----------------------------------------------------------- embed / norm ----
 __global__ void embed_rows_kernel(const uint16_t *E, const int *tok, float *X, int H) {
@@ -29,9 +35,8 @@ __global__ void embed_rows_kernel(const uint16_t *E, const int *tok, float *X, i
     for (int i = threadIdx.x; i < H; i += blockDim.x) X[(size_t)t * H + i] = bf16_to_f32(row[i]);
 }
 
-// A[t] = X[t] / sqrt(mean(X[t]^2) + eps) * g, stored as a hi/lo bf16 pair
-__global__ void rmsnorm_rows_kernel(const float *X, const uint16_t *g, uint16_t *Ahi, uint16_t *Alo, int H,
-                                    float eps) {
+// A[t] = X[t] / sqrt(mean(X[t]^2) + eps) * g, stored as three bf16 terms
+__global__ void rmsnorm_rows_kernel(const float *X, const uint16_t *g, const Terms A, int H, float eps) {
     __shared__ float s_part[32];
     const int t = blockIdx.x;
     const float *x = X + (size_t)t * H;
@@ -44,13 +49,13 @@ __global__ void rmsnorm_rows_kernel(const float *X, const uint16_t *g, uint16_t 
     for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += s_part[w];
     const float rinv = 1.0f / sqrtf(tot / (float)H + eps);
     for (int i = threadIdx.x; i < H; i += blockDim.x)
-        split_store(Ahi, Alo, (size_t)t * H + i, x[i] * rinv * bf16_to_f32(g[i]));
+        split_store(A.p, (size_t)t * H + i, x[i] * rinv * bf16_to_f32(g[i]));
 }
 
 // --------------------------------------------------------------- epilogues ----
 // pair(t, c, a, b): GEMM output row t, columns (c, c + 1)
-struct PEpiQKV {  // packed QKV columns -> Q (bf16 hi/lo) and K/V pages (bf16)
-    uint16_t *Qhi, *Qlo;
+struct PEpiQKV {  // packed QKV columns -> Q (three bf16 terms) and K/V pages (bf16)
+    Terms Q;
     uint16_t *kv;
     const int *pages;
     const float2 *rope;
@@ -72,8 +77,8 @@ struct PEpiQKV {  // packed QKV columns -> Q (bf16 hi/lo) and K/V pages (bf16)
             const float rb = b * cs.x + a * cs.y;
             if (c < qdim) {
                 const size_t qo = (size_t)t * qdim + hd * d + i;
-                split_store(Qhi, Qlo, qo, ra);
-                split_store(Qhi, Qlo, qo + half, rb);
+                split_store(Q.p, qo, ra);
+                split_store(Q.p, qo + half, rb);
             } else {
                 uint16_t *kr = page + ((size_t)(hd - qdim / d) * kPage + slot) * d;
                 kr[i] = f32_to_bf16(ra);
@@ -100,11 +105,11 @@ struct PEpiResidual {  // X[t][c] += v
     }
 };
 
-struct PEpiSwiGLU {  // interleaved (gate, up) columns -> M[t][c/2] = silu(g) * u as hi/lo
-    uint16_t *Mhi, *Mlo;
+struct PEpiSwiGLU {  // interleaved (gate, up) columns -> M[t][c/2] = silu(g) * u as three terms
+    Terms M;
     int ld;
     __device__ void pair(int t, int c, float a, float b) const {
-        split_store(Mhi, Mlo, (size_t)t * ld + (c >> 1), a / (1.0f + expf(-a)) * b);
+        split_store(M.p, (size_t)t * ld + (c >> 1), a / (1.0f + expf(-a)) * b);
     }
 };
 
@@ -182,12 +187,13 @@ static bool encode_kv(CUtensorMap *m, const void *ptr, const Plan &p) {
 
 const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
     const int T = p.max_chunk;
-    bool ok = encode_2d(&m->ahi, b.Ahi, T, p.H, TC_BM) && encode_2d(&m->alo, b.Alo, T, p.H, TC_BM) &&
-              encode_2d(&m->ohi, b.Ohi, T, p.qdim, TC_BM) && encode_2d(&m->olo, b.Olo, T, p.qdim, TC_BM) &&
-              encode_2d(&m->mhi, b.Mhi, T, p.F, TC_BM) && encode_2d(&m->mlo, b.Mlo, T, p.F, TC_BM);
-    if (!ok) return "cuTensorMapEncodeTiled failed for an activation operand";
+    bool ok = true;
     const int tpt = attn_tokens_per_tile(p.group);
-    ok = encode_q(&m->qhi, b.Qhi, p, tpt) && encode_q(&m->qlo, b.Qlo, p, tpt) && encode_kv(&m->kv, b.KV, p);
+    for (int t = 0; t < kTerms; ++t)
+        ok = ok && encode_2d(&m->a[t], b.A[t], T, p.H, TC_BM) && encode_2d(&m->o[t], b.O[t], T, p.qdim, TC_BM) &&
+             encode_2d(&m->m[t], b.M[t], T, p.F, TC_BM) && encode_q(&m->q[t], b.Q[t], p, tpt);
+    if (!ok) return "cuTensorMapEncodeTiled failed for an activation operand";
+    ok = encode_kv(&m->kv, b.KV, p);
     if (!ok) return "cuTensorMapEncodeTiled failed for the attention operands";
     m->wqkv.resize(p.L);
     m->wo.resize(p.L);
@@ -223,8 +229,7 @@ const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
 cudaError_t launch_attn_tc(const Plan &p, const Bufs &b, const PrefillMaps &mp, int layer, int P, int T,
                            cudaStream_t st) {
     AttnArgs a;
-    a.Ohi = b.Ohi;
-    a.Olo = b.Olo;
+    for (int t = 0; t < kTerms; ++t) a.O[t] = b.O[t];
     a.pages = b.pages;
     a.err = b.ctrl + CTRL_ERR;
     a.P = P;
@@ -237,18 +242,20 @@ cudaError_t launch_attn_tc(const Plan &p, const Bufs &b, const PrefillMaps &mp, 
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)p.d);
     dim3 grid((T + a.tpt - 1) / a.tpt, p.nkv);
     if (p.d == 128)
-        attn_tc_kernel<128><<<grid, AT_THREADS, AttnSmem<128>::TOTAL + 1024, st>>>(mp.qhi, mp.qlo, mp.kv, a);
+        attn_tc_kernel<128><<<grid, AT_THREADS, AttnSmem<128>::TOTAL + 1024, st>>>(mp.q[0], mp.q[1], mp.q[2], mp.kv,
+                                                                                  a);
     else
-        attn_tc_kernel<64><<<grid, AT_THREADS, AttnSmem<64>::TOTAL + 1024, st>>>(mp.qhi, mp.qlo, mp.kv, a);
+        attn_tc_kernel<64><<<grid, AT_THREADS, AttnSmem<64>::TOTAL + 1024, st>>>(mp.q[0], mp.q[1], mp.q[2], mp.kv,
+                                                                                a);
     return cudaGetLastError();
 }
 
 template <class Epi>
-static cudaError_t gemm(const CUtensorMap &ahi, const CUtensorMap &alo, const CUtensorMap &w, int T, int N, int K,
-                        int *err, const Epi &epi, cudaStream_t st, LaunchHook *hook, const char *name) {
+static cudaError_t gemm(const CUtensorMap *a, const CUtensorMap &w, int T, int N, int K, int *err, const Epi &epi,
+                        cudaStream_t st, LaunchHook *hook, const char *name) {
     if (hook) hook->before(name);
-    dim3 grid((N + TC_BN - 1) / TC_BN, (T + TC_BM - 1) / TC_BM);
-    gemm_tc_kernel<Epi><<<grid, TC_THREADS, TC_SMEM, st>>>(ahi, alo, w, T, N, K, err, epi);
+    dim3 grid((T + TC_BM - 1) / TC_BM, (N + TC_BN - 1) / TC_BN);
+    gemm_tc_kernel<Epi><<<grid, TC_THREADS, TC_SMEM, st>>>(a[0], a[1], a[2], w, T, N, K, err, epi);
     if (hook) hook->after(name);
     return cudaGetLastError();
 }
@@ -263,10 +270,11 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         const LayerOffsets &lo = p.layer[l];
         uint16_t *kvl = b.KV + (size_t)l * p.kv_layer_elems;
         // A3 + A4: RMSNorm, QKV (+bias), RoPE, paged KV append
-        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.attn_norm, b.Ahi, b.Alo, p.H, p.cfg.rms_eps);
-        PEpiQKV eq = {b.Qhi, b.Qlo, kvl, b.pages, b.rope, p.cfg.qkv_bias ? b.W + lo.bqkv : nullptr, P, p.qdim,
+        const Terms A = {{b.A[0], b.A[1], b.A[2]}};
+        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.attn_norm, A, p.H, p.cfg.rms_eps);
+        PEpiQKV eq = {{{b.Q[0], b.Q[1], b.Q[2]}}, kvl, b.pages, b.rope, p.cfg.qkv_bias ? b.W + lo.bqkv : nullptr, P, p.qdim,
                       p.kvdim, p.d, p.nkv, p.kv_page_elems};
-        if ((e = gemm(mp.ahi, mp.alo, mp.wqkv[l], T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
+        if ((e = gemm(mp.a, mp.wqkv[l], T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
             return e;
         // A5: causal attention over the cache (earlier chunks + this one), tensor cores
         if (hook) hook->before("prefill_attention");
@@ -274,16 +282,17 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         if (hook) hook->after("prefill_attention");
         if (e != cudaSuccess) return e;
         // A6: O projection + residual
-        if ((e = gemm(mp.ohi, mp.olo, mp.wo[l], T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
+        if ((e = gemm(mp.o, mp.wo[l], T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_o_proj")) != cudaSuccess)
             return e;
         // A7: RMSNorm + gate/up + SwiGLU
-        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.ffn_norm, b.Ahi, b.Alo, p.H, p.cfg.rms_eps);
-        if ((e = gemm(mp.ahi, mp.alo, mp.wgu[l], T, 2 * p.F, p.H, err, PEpiSwiGLU{b.Mhi, b.Mlo, p.F}, st, hook,
+        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.ffn_norm, A, p.H, p.cfg.rms_eps);
+        const Terms M = {{b.M[0], b.M[1], b.M[2]}};
+        if ((e = gemm(mp.a, mp.wgu[l], T, 2 * p.F, p.H, err, PEpiSwiGLU{M, p.F}, st, hook,
                       "prefill_gate_up")) != cudaSuccess)
             return e;
         // A8: down projection + residual
-        if ((e = gemm(mp.mhi, mp.mlo, mp.wd[l], T, p.H, p.F, err, PEpiResidual{b.X, p.H}, st, hook,
+        if ((e = gemm(mp.m, mp.wd[l], T, p.H, p.F, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_down")) != cudaSuccess)
             return e;
     }

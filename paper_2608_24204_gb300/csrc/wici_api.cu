@@ -129,14 +129,12 @@ const char *wici::make_plan(const wici_config *cfg, int num_sms, Plan *p) {
     P.ws_pages = ws((size_t)P.max_pages * 4);
     P.ws_tok = ws(T * 4);
     P.ws_X = ws(T * H * 4);
-    P.ws_Qhi = ws(T * P.qdim * 2);
-    P.ws_Qlo = ws(T * P.qdim * 2);
-    P.ws_Ahi = ws(T * H * 2);
-    P.ws_Alo = ws(T * H * 2);
-    P.ws_Ohi = ws(T * P.qdim * 2);
-    P.ws_Olo = ws(T * P.qdim * 2);
-    P.ws_Mhi = ws(T * F * 2);
-    P.ws_Mlo = ws(T * F * 2);
+    for (int t = 0; t < kTerms; ++t) {
+        P.ws_Q[t] = ws(T * P.qdim * 2);
+        P.ws_A[t] = ws(T * H * 2);
+        P.ws_O[t] = ws(T * P.qdim * 2);
+        P.ws_M[t] = ws(T * F * 2);
+    }
     P.ws_bytes = w;
     return nullptr;
 }
@@ -158,14 +156,12 @@ static Bufs make_bufs(const Plan &p, void *W, void *KV, void *WS) {
     b.pages = (int *)(ws + p.ws_pages);
     b.tok = (int *)(ws + p.ws_tok);
     b.X = (float *)(ws + p.ws_X);
-    b.Qhi = (uint16_t *)(ws + p.ws_Qhi);
-    b.Qlo = (uint16_t *)(ws + p.ws_Qlo);
-    b.Ahi = (uint16_t *)(ws + p.ws_Ahi);
-    b.Alo = (uint16_t *)(ws + p.ws_Alo);
-    b.Ohi = (uint16_t *)(ws + p.ws_Ohi);
-    b.Olo = (uint16_t *)(ws + p.ws_Olo);
-    b.Mhi = (uint16_t *)(ws + p.ws_Mhi);
-    b.Mlo = (uint16_t *)(ws + p.ws_Mlo);
+    for (int t = 0; t < kTerms; ++t) {
+        b.Q[t] = (uint16_t *)(ws + p.ws_Q[t]);
+        b.A[t] = (uint16_t *)(ws + p.ws_A[t]);
+        b.O[t] = (uint16_t *)(ws + p.ws_O[t]);
+        b.M[t] = (uint16_t *)(ws + p.ws_M[t]);
+    }
     return b;
 }
 
