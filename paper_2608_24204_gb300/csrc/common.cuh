@@ -119,6 +119,12 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
         : "memory");
 }
 
+// Start moving `bytes` of global memory into L2, with no destination and nothing
+// to wait for (16-byte aligned address and size).
+__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 // L2 policy for data read exactly once per step (weights): evict first.
 __device__ __forceinline__ uint64_t l2_evict_first() {
     uint64_t p;

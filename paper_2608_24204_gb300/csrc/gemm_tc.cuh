@@ -3,7 +3,7 @@
 //   C[T][N] = (A_0 + A_1 + A_2)[T][K] . W[N][K]^T,  fp32 accumulation in TMEM
 //
 // A is an fp32 activation carried as kTerms = 3 bf16 terms (split_bf16x3); W is
-// bf16 and exact.  The three products accumulate into one 128x256 fp32
+// bf16 and exact.  The three products accumulate into one 128x128 fp32
 // accumulator, so the activations keep fp32 precision on bf16 MMAs (the bf16x3
 // scheme of Henry, Tang & Heinecke, ARITH 2019, applied to one operand).
 //

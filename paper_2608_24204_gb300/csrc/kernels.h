@@ -23,6 +23,7 @@ struct Bufs {
     float *m;         // decode SwiGLU output                               [F]
     float *logits;    // last logits                                        [V]
     int2 *amax;       // per-CTA argmax partials (value bits, index)        [num_sms]
+    float *fd_part;   // flash-decode split states                           [nkv][splits][group][d + 4]
     float2 *rope;     // (cos, sin) of p * theta^(-2i/d)                     [max_tokens][d/2]
     int *pages;       // logical -> physical KV page                         [max_pages]
     int *tok;         // prefill chunk tokens                                [max_chunk]
@@ -51,6 +52,11 @@ struct LaunchHook {
     virtual void after(const char *name) = 0;
     virtual ~LaunchHook() {}
 };
+
+// Flash-decode split count for a context of max_pages pages, and the floats
+// of its split-state buffer.
+int fd_splits(int max_pages);
+size_t fd_part_floats(int nkv, int group, int d, int max_pages);
 
 // One-time per-process kernel attributes (dynamic shared memory limits).
 cudaError_t setup_kernels();

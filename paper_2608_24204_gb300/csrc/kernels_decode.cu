@@ -31,6 +31,10 @@ struct GemvIn {
     float *x_out;           // embed variant: CTA 0 stores the embedded row here
     int *ctrl;
     float eps;
+    // the GEMV launched after this one: the producer moves the first rows of
+    // this CTA's share of it into L2 once its own rows are issued
+    const uint16_t *next_W;  // nullptr: none
+    int next_K, next_n_units, next_rpu;
 };
 
 // ---------------------------------------------------------------- epilogues --
@@ -225,6 +229,18 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const GemvIn g, c
                 bulk_g2s(ring0 + slot * g.slot_bytes, src + (size_t)s * RPS * g.K, bytes, full0 + 8 * slot, pol);
                 issued = s + 1;
             }
+            if (g.next_W) {
+                // the next kernel's CTA of the same index streams units [nu0, nu1); its
+                // first ring-full is fetched while this CTA drains, so the HBM stays busy
+                // across the kernel boundary
+                const int nu0 = (int)(((long long)blockIdx.x * g.next_n_units) / G);
+                const int nu1 = (int)(((long long)(blockIdx.x + 1) * g.next_n_units) / G);
+                const size_t total = (size_t)(nu1 - nu0) * g.next_rpu * g.next_K * 2;
+                const size_t want = total < (size_t)kGemvRingBytes ? total : (size_t)kGemvRingBytes;
+                const uint8_t *src = reinterpret_cast<const uint8_t *>(g.next_W + (size_t)nu0 * g.next_rpu * g.next_K);
+                for (size_t off = 0; off < want; off += 32768)
+                    bulk_prefetch_l2(src + off, (uint32_t)(want - off < 32768 ? want - off : 32768));
+            }
             // no copy may still be landing in this CTA's shared memory when it exits
             for (int s = max(0, issued - S); s < issued; ++s)
                 mbar_wait(full0 + 8 * (s % S), (s / S) & 1, err, SITE_GEMV_DRAIN);
@@ -398,18 +414,26 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_kernel(const GemvIn g, c
 }
 
 // ------------------------------------------------------------ flash-decode ----
-// Grid (kFdSplits, nkv) in clusters of kFdSplits CTAs: one cluster per KV head g,
-// CTA rank r covering a contiguous range of the cached pages.  Block = group x
-// wph query warps + 1 producer warp.  The producer streams the range's pages (the
-// K and V blocks of head g, 16 x d bf16 each, contiguous in a page) through a
-// kFdStages-slot TMA ring; query warp (j, set) runs an online softmax for query
-// head g*group + j over the pages i = set (mod wph) of the range.  The length
-// comes from the device position, so one captured graph serves every step.  The
-// wph states of a head are merged in shared memory, then the CTA of rank 0
-// combines the kFdSplits CTAs' partials over distributed shared memory, in rank
-// order.
-constexpr int kFdStages = 8;
-constexpr int kFdSplits = 16;   // cluster size (non-portable: 16 > 8)
+// Split-K attention of one query token over the paged cache (Sec. 5.1 decode
+// step).  Grid (S, nkv): CTA (r, g) covers split r of KV head g, a contiguous
+// range of the cached pages; block = group x wph query warps + 1 producer warp.
+// The producer streams the range's pages (the K and V blocks of head g, 16 x d
+// bf16 each, contiguous in a page) through a small TMA ring; query warp
+// (j, set) runs an online softmax for query head g*group + j over the pages
+// i = set (mod wph) of the range, and the wph states of a head are merged in
+// shared memory.  Each CTA writes its per-head state (acc, m, l) to global
+// memory and takes a ticket; the last CTA of head g combines the splits in
+// split order, so the result does not depend on which CTA finishes last.
+//
+// No cluster and a small footprint (<= 288 threads, 32 KB ring): the CTAs fit
+// beside a GEMV CTA on the same SM, so under programmatic dependent launch the
+// kernel starts streaming pages while the QKV GEMV still runs, and the O
+// projection's weight ring fills while the attention finishes.  The length comes
+// from the device position, so one captured graph serves every step; the split
+// count adapts to it at run time (at most gridDim.x splits).
+constexpr uint32_t kFdRingBytes = 32768;
+constexpr int kFdMaxQueryWarps = 8;
+constexpr int kFdMaxSplits = 32;
 
 struct FDArgs {
     const float *q;
@@ -417,38 +441,13 @@ struct FDArgs {
     const int *pages;
     int *ctrl;
     float *o;
+    float *part;         // [nkv][splits][group][d + 4]: acc[d], m, l of each split
     int nkv, group, wph;
     size_t page_elems;
     float qscale;        // log2(e) / sqrt(d)
 };
 
 enum : int { SITE_FD_EMPTY = 31, SITE_FD_FULL = 32, SITE_FD_DRAIN = 33 };
-
-__device__ __forceinline__ uint32_t cluster_ctarank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-__device__ __forceinline__ void cluster_sync_all() {
-    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-__device__ __forceinline__ uint32_t dsmem_addr(const void *local, uint32_t rank) {
-    uint32_t r;
-    asm("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(local)), "r"(rank));
-    return r;
-}
-// plain (reorderable) loads from another CTA's shared memory; ordering against
-// the writes comes from the cluster barrier that precedes them
-__device__ __forceinline__ float2 ld_dsmem2(uint32_t addr) {
-    float2 v;
-    asm("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr));
-    return v;
-}
-__device__ __forceinline__ float4 ld_dsmem4(uint32_t addr) {
-    float4 v;
-    asm("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
-    return v;
-}
 
 // (m, l, acc) online-softmax merge of b into a (log2 domain)
 // An empty state (no keys seen) has m = -inf, l = 0, acc = 0 and is skipped:
@@ -472,19 +471,32 @@ __device__ __forceinline__ void fd_merge(float &m, float &l, float *acc, float m
 }
 
 template <int D>
-__global__ void __launch_bounds__(544, 2) flash_decode_kernel(const FDArgs a) {
+__global__ void __launch_bounds__(32 * (kFdMaxQueryWarps + 1)) flash_decode_kernel(const FDArgs a) {
     constexpr int EPL = D / 32;
-    constexpr uint32_t BLK = kPage * D * 2;     // bytes of one K (or V) block of a page
-    extern __shared__ __align__(128) uint8_t fsm[];   // [kFdStages][K block | V block]
-    __shared__ __align__(8) uint64_t full_bar[kFdStages], empty_bar[kFdStages];
-    __shared__ __align__(16) float s_state[16][D + 4];   // per query warp: acc[D], m, l
+    constexpr uint32_t BLK = kPage * D * 2;              // bytes of one K (or V) block of a page
+    constexpr int STAGES = (int)(kFdRingBytes / (2 * BLK));
+    constexpr int STRIDE = D + 4;                        // floats per state: acc[D], m, l, pad
+    extern __shared__ __align__(128) uint8_t fsm[];      // [STAGES][K block | V block]
+    __shared__ __align__(8) uint64_t full_bar[STAGES], empty_bar[STAGES];
+    __shared__ __align__(16) float s_state[kFdMaxQueryWarps][STRIDE];
+    __shared__ int s_last;
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nq = a.group * a.wph;   // query warps
     const int g = blockIdx.y;
-    const uint32_t rank = cluster_ctarank();
+    const int r = blockIdx.x;
     int *err = a.ctrl + CTRL_ERR;
+
+    // the position is only advanced at the end of a step, so it is stable here
+    const int len = *reinterpret_cast<volatile int *>(a.ctrl + CTRL_POS) + 1;
+    const int npages = (len + kPage - 1) / kPage;
+    const int pps = (npages + (int)gridDim.x - 1) / (int)gridDim.x;
+    const int splits = (npages + pps - 1) / pps;          // every split below this has pages
+    if (r >= splits) return;                              // idle CTA: no state, no ticket
+    const int p0 = r * pps;
+    const int n = min(npages, p0 + pps) - p0;
+
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kFdStages; ++s) {
+        for (int s = 0; s < STAGES; ++s) {
             mbar_init(smem_u32(&full_bar[s]), 1);
             mbar_init(smem_u32(&empty_bar[s]), a.group);
         }
@@ -492,13 +504,6 @@ __global__ void __launch_bounds__(544, 2) flash_decode_kernel(const FDArgs a) {
     }
     __syncthreads();
     griddep_launch_dependents();
-
-    // the position is only advanced at the end of a step, so it is stable here
-    const int len = *reinterpret_cast<volatile int *>(a.ctrl + CTRL_POS) + 1;
-    const int npages = (len + kPage - 1) / kPage;
-    const int pps = (npages + kFdSplits - 1) / kFdSplits;
-    const int p0 = (int)rank * pps;
-    const int n = max(0, min(npages, p0 + pps) - p0);
 
     if (w == nq) {  // ---------------------------------------------- producer
         // the whole warp walks the pages so that 32 page-table entries are read at
@@ -509,10 +514,10 @@ __global__ void __launch_bounds__(544, 2) flash_decode_kernel(const FDArgs a) {
         for (int i = 0; i < n; ++i) {
             if ((i & 31) == 0 && i + lane < n) my_page = a.pages[p0 + i + lane];
             const int page = __shfl_sync(0xffffffffu, my_page, i & 31);
-            const int s = i % kFdStages;
+            const int s = i % STAGES;
             bool ok = true;
-            if (lane == 0 && i >= kFdStages)
-                ok = mbar_wait(smem_u32(&empty_bar[s]), ((i / kFdStages) + 1) & 1, err, SITE_FD_EMPTY);
+            if (lane == 0 && i >= STAGES)
+                ok = mbar_wait(smem_u32(&empty_bar[s]), ((i / STAGES) + 1) & 1, err, SITE_FD_EMPTY);
             if (!__shfl_sync(0xffffffffu, (int)ok, 0)) break;
             // the page holding the current position is written by the preceding kernel
             if (!waited && p0 + i == npages - 1) {
@@ -530,103 +535,107 @@ __global__ void __launch_bounds__(544, 2) flash_decode_kernel(const FDArgs a) {
             issued = i + 1;
         }
         if (lane == 0)
-            for (int i = max(0, issued - kFdStages); i < issued; ++i)
-                mbar_wait(smem_u32(&full_bar[i % kFdStages]), (i / kFdStages) & 1, err, SITE_FD_DRAIN);
+            for (int i = max(0, issued - STAGES); i < issued; ++i)
+                mbar_wait(smem_u32(&full_bar[i % STAGES]), (i / STAGES) & 1, err, SITE_FD_DRAIN);
         __syncwarp();
-    } else {  // ------------------------------------------------- query warps
-        griddep_wait();
-        const int j = w % a.group, set = w / a.group;
-        const int head = g * a.group + j;
-        float qv[EPL], acc[EPL];
-        if constexpr (EPL == 4) {
-            const float4 q4 = *reinterpret_cast<const float4 *>(a.q + head * D + lane * 4);
-            qv[0] = q4.x * a.qscale; qv[1] = q4.y * a.qscale; qv[2] = q4.z * a.qscale; qv[3] = q4.w * a.qscale;
-        } else {
-            const float2 q2 = *reinterpret_cast<const float2 *>(a.q + head * D + lane * 2);
-            qv[0] = q2.x * a.qscale; qv[1] = q2.y * a.qscale;
+        return;   // the producer takes no part in the named barriers below
+    }
+
+    // ------------------------------------------------------------ query warps
+    griddep_wait();
+    const int j = w % a.group, set = w / a.group;
+    const int head = g * a.group + j;
+    float qv[EPL], acc[EPL];
+    if constexpr (EPL == 4) {
+        const float4 q4 = *reinterpret_cast<const float4 *>(a.q + head * D + lane * 4);
+        qv[0] = q4.x * a.qscale; qv[1] = q4.y * a.qscale; qv[2] = q4.z * a.qscale; qv[3] = q4.w * a.qscale;
+    } else {
+        const float2 q2 = *reinterpret_cast<const float2 *>(a.q + head * D + lane * 2);
+        qv[0] = q2.x * a.qscale; qv[1] = q2.y * a.qscale;
+    }
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
+    float m = -INFINITY, l = 0.f;
+    const int key = lane >> 1;   // the key whose score this lane ends with
+    bool ok = true;
+    for (int i = set; i < n && ok; i += a.wph) {
+        const int s = i % STAGES;
+        ok = mbar_wait(smem_u32(&full_bar[s]), (i / STAGES) & 1, err, SITE_FD_FULL);
+        if (!ok) break;
+        const uint8_t *Ks = fsm + (size_t)s * 2 * BLK;
+        const uint8_t *Vs = Ks + BLK;
+        const int ntok = min(kPage, len - (p0 + i) * kPage);
+        // partial dot products of this lane's d-slice with the 16 keys
+        float sc[kPage];
+#pragma unroll
+        for (int t = 0; t < kPage; ++t) {
+            const uint8_t *kr = Ks + (t * D + lane * EPL) * 2;
+            if constexpr (EPL == 4) {
+                const uint2 kw = *reinterpret_cast<const uint2 *>(kr);
+                sc[t] = qv[0] * bf16lo(kw.x) + qv[1] * bf16hi(kw.x) + qv[2] * bf16lo(kw.y) + qv[3] * bf16hi(kw.y);
+            } else {
+                const uint32_t kw = *reinterpret_cast<const uint32_t *>(kr);
+                sc[t] = qv[0] * bf16lo(kw) + qv[1] * bf16hi(kw);
+            }
         }
+        // transposed butterfly: lanes 2k and 2k+1 end with the full score of key k
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
-        float m = -INFINITY, l = 0.f;
-        const int key = lane >> 1;   // the key whose score this lane ends with
-        bool ok = true;
-        for (int i = set; i < n && ok; i += a.wph) {
-            const int s = i % kFdStages;
-            ok = mbar_wait(smem_u32(&full_bar[s]), (i / kFdStages) & 1, err, SITE_FD_FULL);
-            if (!ok) break;
-            const uint8_t *Ks = fsm + (size_t)s * 2 * BLK;
-            const uint8_t *Vs = Ks + BLK;
-            const int ntok = min(kPage, len - (p0 + i) * kPage);
-            // partial dot products of this lane's d-slice with the 16 keys
-            float sc[kPage];
+        for (int o = 16, cnt = kPage; o > 0; o >>= 1) {
+            if (cnt > 1) {
+                const bool up = (lane & o) != 0;
 #pragma unroll
-            for (int t = 0; t < kPage; ++t) {
-                const uint8_t *kr = Ks + (t * D + lane * EPL) * 2;
-                if constexpr (EPL == 4) {
-                    const uint2 kw = *reinterpret_cast<const uint2 *>(kr);
-                    sc[t] = qv[0] * bf16lo(kw.x) + qv[1] * bf16hi(kw.x) + qv[2] * bf16lo(kw.y) + qv[3] * bf16hi(kw.y);
-                } else {
-                    const uint32_t kw = *reinterpret_cast<const uint32_t *>(kr);
-                    sc[t] = qv[0] * bf16lo(kw) + qv[1] * bf16hi(kw);
+                for (int t = 0; t < cnt / 2; ++t) {
+                    const float send = up ? sc[t] : sc[t + cnt / 2];
+                    const float keep = up ? sc[t + cnt / 2] : sc[t];
+                    sc[t] = keep + __shfl_xor_sync(0xffffffffu, send, o);
                 }
+                cnt >>= 1;
+            } else {
+                sc[0] += __shfl_xor_sync(0xffffffffu, sc[0], o);
             }
-            // transposed butterfly: lanes 2k and 2k+1 end with the full score of key k
-#pragma unroll
-            for (int o = 16, cnt = kPage; o > 0; o >>= 1) {
-                if (cnt > 1) {
-                    const bool up = (lane & o) != 0;
-#pragma unroll
-                    for (int t = 0; t < cnt / 2; ++t) {
-                        const float send = up ? sc[t] : sc[t + cnt / 2];
-                        const float keep = up ? sc[t + cnt / 2] : sc[t];
-                        sc[t] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-                    }
-                    cnt >>= 1;
-                } else {
-                    sc[0] += __shfl_xor_sync(0xffffffffu, sc[0], o);
-                }
-            }
-            const float my = key < ntok ? sc[0] : -INFINITY;   // slots past the length are masked
-            const float mx = fmaxf(m, warp_max(my));
-            const float corr = exp2f(m - mx);
-            const float pme = exp2f(my - mx);                  // 0 for masked keys
-            l = l * corr + pme;   // per-lane share of the denominator (every key is held by two lanes)
-#pragma unroll
-            for (int e = 0; e < EPL; ++e) acc[e] *= corr;
-#pragma unroll
-            for (int t = 0; t < kPage; ++t) {
-                // slots past the length are never used: unwritten cache memory may hold NaN bits
-                const bool valid = t < ntok;
-                const float pt = __shfl_sync(0xffffffffu, pme, 2 * t);
-                const uint8_t *vr = Vs + (t * D + lane * EPL) * 2;
-                if constexpr (EPL == 4) {
-                    uint2 vw = *reinterpret_cast<const uint2 *>(vr);
-                    if (!valid) vw = make_uint2(0u, 0u);
-                    acc[0] = fmaf(pt, bf16lo(vw.x), acc[0]);
-                    acc[1] = fmaf(pt, bf16hi(vw.x), acc[1]);
-                    acc[2] = fmaf(pt, bf16lo(vw.y), acc[2]);
-                    acc[3] = fmaf(pt, bf16hi(vw.y), acc[3]);
-                } else {
-                    uint32_t vw = *reinterpret_cast<const uint32_t *>(vr);
-                    if (!valid) vw = 0u;
-                    acc[0] = fmaf(pt, bf16lo(vw), acc[0]);
-                    acc[1] = fmaf(pt, bf16hi(vw), acc[1]);
-                }
-            }
-            m = mx;
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&empty_bar[s]));
         }
-        l = warp_sum(l) * 0.5f;
+        const float my = key < ntok ? sc[0] : -INFINITY;   // slots past the length are masked
+        const float mx = fmaxf(m, warp_max(my));
+        const float corr = exp2f(m - mx);
+        const float pme = exp2f(my - mx);                  // 0 for masked keys
+        l = l * corr + pme;   // per-lane share of the denominator (every key is held by two lanes)
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) acc[e] *= corr;
+#pragma unroll
+        for (int t = 0; t < kPage; ++t) {
+            // slots past the length are never used: they may hold stale values
+            const bool valid = t < ntok;
+            const float pt = __shfl_sync(0xffffffffu, pme, 2 * t);
+            const uint8_t *vr = Vs + (t * D + lane * EPL) * 2;
+            if constexpr (EPL == 4) {
+                uint2 vw = *reinterpret_cast<const uint2 *>(vr);
+                if (!valid) vw = make_uint2(0u, 0u);
+                acc[0] = fmaf(pt, bf16lo(vw.x), acc[0]);
+                acc[1] = fmaf(pt, bf16hi(vw.x), acc[1]);
+                acc[2] = fmaf(pt, bf16lo(vw.y), acc[2]);
+                acc[3] = fmaf(pt, bf16hi(vw.y), acc[3]);
+            } else {
+                uint32_t vw = *reinterpret_cast<const uint32_t *>(vr);
+                if (!valid) vw = 0u;
+                acc[0] = fmaf(pt, bf16lo(vw), acc[0]);
+                acc[1] = fmaf(pt, bf16hi(vw), acc[1]);
+            }
+        }
+        m = mx;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&empty_bar[s]));
+    }
+    l = warp_sum(l) * 0.5f;
+    if (a.wph > 1) {
 #pragma unroll
         for (int e = 0; e < EPL; ++e) s_state[w][lane * EPL + e] = acc[e];
         if (lane == 0) {
             s_state[w][D] = m;
             s_state[w][D + 1] = l;
         }
-        // merge the wph page sets of each head into set 0's slot (fixed set order)
+        // merge the wph page sets of each head into set 0 (fixed set order)
         asm volatile("bar.sync 1, %0;" ::"r"(32 * nq) : "memory");
-        if (set == 0) {
+        if (set == 0)
             for (int t = 1; t < a.wph; ++t) {
                 const float *o = s_state[t * a.group + j];
                 float ob[EPL];
@@ -634,58 +643,66 @@ __global__ void __launch_bounds__(544, 2) flash_decode_kernel(const FDArgs a) {
                 for (int e = 0; e < EPL; ++e) ob[e] = o[lane * EPL + e];
                 fd_merge<EPL>(m, l, acc, o[D], o[D + 1], ob);
             }
-            // all reads of the other sets' states are done before set 0 overwrites its own
-            __syncwarp();
+    }
+    // this split's state of head j -> global; then the ticket
+    float *mine = a.part + ((size_t)(g * gridDim.x + r) * a.group + j) * STRIDE;
+    if (set == 0) {
+        if constexpr (EPL == 4)
+            *reinterpret_cast<float4 *>(mine + lane * 4) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+        else
+            *reinterpret_cast<float2 *>(mine + lane * 2) = make_float2(acc[0], acc[1]);
+        if (lane == 0) *reinterpret_cast<float2 *>(mine + D) = make_float2(m, l);
+        __threadfence();
+    }
+    asm volatile("bar.sync 1, %0;" ::"r"(32 * nq) : "memory");
+    if (threadIdx.x == 0) {
+        const int t = atomicAdd(a.ctrl + CTRL_ATTN_TICKET0 + g, 1);
+        s_last = (t == splits - 1);
+    }
+    asm volatile("bar.sync 1, %0;" ::"r"(32 * nq) : "memory");
+    if (!s_last || set != 0) return;
+
+    // ------------------------------------------- last CTA of head g: combine
+    __threadfence();
+    const float *base = a.part + ((size_t)g * gridDim.x * a.group + j) * STRIDE;
+    const size_t sstride = (size_t)a.group * STRIDE;     // floats between splits of one head
+    float2 ml = make_float2(-INFINITY, 0.f);
+    if (lane < splits) ml = __ldcg(reinterpret_cast<const float2 *>(base + lane * sstride + D));
+    const float M = warp_max(ml.x);
+    const float f = lane < splits ? exp2f(ml.x - M) : 0.f;
+    const float L = warp_sum(ml.y * f);
+    float out[EPL];
 #pragma unroll
-            for (int e = 0; e < EPL; ++e) s_state[j][lane * EPL + e] = acc[e];
-            if (lane == 0) {
-                s_state[j][D] = m;
-                s_state[j][D + 1] = l;
+    for (int e = 0; e < EPL; ++e) out[e] = 0.f;
+    for (int s0 = 0; s0 < splits; s0 += 8) {
+        float v[8][EPL];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int sp = min(s0 + u, splits - 1);
+            const float *src = base + sp * sstride + lane * EPL;
+            if constexpr (EPL == 4) {
+                const float4 t4 = __ldcg(reinterpret_cast<const float4 *>(src));
+                v[u][0] = t4.x; v[u][1] = t4.y; v[u][2] = t4.z; v[u][3] = t4.w;
+            } else {
+                const float2 t2 = __ldcg(reinterpret_cast<const float2 *>(src));
+                v[u][0] = t2.x; v[u][1] = t2.y;
             }
         }
-    }
-    cluster_sync_all();   // every CTA's merged partials are written and visible to the cluster
-    if (rank == 0 && w < a.group) {
-        const int head = g * a.group + w;
-        // lanes 0..15 read the (m, l) of one split each
-        float2 ml = make_float2(-INFINITY, 0.f);
-        if (lane < kFdSplits) ml = ld_dsmem2(dsmem_addr(&s_state[w][D], lane));
-        const float M = warp_max(ml.x);
-        const float f = lane < kFdSplits ? exp2f(ml.x - M) : 0.f;   // empty splits: exp2(-inf) = 0
-        const float L = warp_sum(ml.y * f);
-        float out[EPL];
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) out[e] = 0.f;
-        if constexpr (EPL == 4) {
-            float4 v[kFdSplits];
+        for (int u = 0; u < 8; ++u) {
+            const float fs = __shfl_sync(0xffffffffu, f, (s0 + u) & 31);
+            if (s0 + u < splits)
 #pragma unroll
-            for (int s = 0; s < kFdSplits; ++s) v[s] = ld_dsmem4(dsmem_addr(&s_state[w][lane * 4], (uint32_t)s));
-#pragma unroll
-            for (int s = 0; s < kFdSplits; ++s) {
-                const float fs = __shfl_sync(0xffffffffu, f, s);
-                out[0] = fmaf(v[s].x, fs, out[0]);
-                out[1] = fmaf(v[s].y, fs, out[1]);
-                out[2] = fmaf(v[s].z, fs, out[2]);
-                out[3] = fmaf(v[s].w, fs, out[3]);
-            }
-            const float inv = 1.0f / L;
-            *reinterpret_cast<float4 *>(a.o + head * D + lane * 4) =
-                make_float4(out[0] * inv, out[1] * inv, out[2] * inv, out[3] * inv);
-        } else {
-            float2 v[kFdSplits];
-#pragma unroll
-            for (int s = 0; s < kFdSplits; ++s) v[s] = ld_dsmem2(dsmem_addr(&s_state[w][lane * 2], (uint32_t)s));
-#pragma unroll
-            for (int s = 0; s < kFdSplits; ++s) {
-                const float fs = __shfl_sync(0xffffffffu, f, s);
-                out[0] = fmaf(v[s].x, fs, out[0]);
-                out[1] = fmaf(v[s].y, fs, out[1]);
-            }
-            const float inv = 1.0f / L;
-            *reinterpret_cast<float2 *>(a.o + head * D + lane * 2) = make_float2(out[0] * inv, out[1] * inv);
+                for (int e = 0; e < EPL; ++e) out[e] = fmaf(v[u][e], fs, out[e]);
         }
     }
-    cluster_sync_all();   // keep every CTA's shared memory alive until rank 0 has read it
+    const float inv = 1.0f / L;
+    if constexpr (EPL == 4)
+        *reinterpret_cast<float4 *>(a.o + head * D + lane * 4) =
+            make_float4(out[0] * inv, out[1] * inv, out[2] * inv, out[3] * inv);
+    else
+        *reinterpret_cast<float2 *>(a.o + head * D + lane * 2) = make_float2(out[0] * inv, out[1] * inv);
+    if (j == 0 && lane == 0) a.ctrl[CTRL_ATTN_TICKET0 + g] = 0;   // ready for the next layer
 }
 
 // ------------------------------------------------------------ probe kernel ----
@@ -717,27 +734,23 @@ static cudaError_t launch(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStr
     return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
-// query warps per head: up to 4, at most 16 query warps per CTA (two CTAs fit an SM,
-// so a 16-CTA cluster needs only 8 SMs of a GPC)
-static int fd_wph(int group) { return group >= 4 ? 16 / group : 4; }
+// query warps per head: at most kFdMaxQueryWarps query warps per CTA
+static int fd_wph(int group) { return group >= kFdMaxQueryWarps ? 1 : kFdMaxQueryWarps / group; }
+
+int fd_splits(int max_pages) {
+    const int s = (max_pages + 3) / 4;   // about four pages per split at the largest length
+    return s < 1 ? 1 : (s > kFdMaxSplits ? kFdMaxSplits : s);
+}
+
+size_t fd_part_floats(int nkv, int group, int d, int max_pages) {
+    return (size_t)nkv * fd_splits(max_pages) * group * (d + 4);
+}
 
 template <int D>
 static cudaError_t launch_fd(const Plan &p, const FDArgs &fa, cudaStream_t st, bool pdl) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(kFdSplits, p.nkv);
-    cfg.blockDim = dim3(32 * (fa.group * fa.wph + 1));
-    cfg.dynamicSmemBytes = (size_t)kFdStages * 2 * kPage * D * 2;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[2];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
-    attr[1].id = cudaLaunchAttributeClusterDimension;
-    attr[1].val.clusterDim.x = kFdSplits;
-    attr[1].val.clusterDim.y = 1;
-    attr[1].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, flash_decode_kernel<D>, fa);
+    constexpr uint32_t BLK = kPage * D * 2;
+    return launch(flash_decode_kernel<D>, dim3(fd_splits(p.max_pages), p.nkv), dim3(32 * (fa.group * fa.wph + 1)),
+                  (size_t)(kFdRingBytes / (2 * BLK)) * 2 * BLK, st, pdl, fa);
 }
 
 // the (NCH, RPS, FULL) shapes of every supported K (K % 8 == 0, K <= 16384)
@@ -773,18 +786,6 @@ static cudaError_t set_gemv_attrs() {
 
 cudaError_t setup_kernels() {
     cudaError_t e;
-    if ((e = cudaFuncSetAttribute(flash_decode_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
-        cudaSuccess)
-        return e;
-    if ((e = cudaFuncSetAttribute(flash_decode_kernel<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) !=
-        cudaSuccess)
-        return e;
-    if ((e = cudaFuncSetAttribute(flash_decode_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  kFdStages * 2 * kPage * 128 * 2)) != cudaSuccess)
-        return e;
-    if ((e = cudaFuncSetAttribute(flash_decode_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  kFdStages * 2 * kPage * 64 * 2)) != cudaSuccess)
-        return e;
     if ((e = set_gemv_attrs<EpiResidual>()) != cudaSuccess) return e;
     if ((e = set_gemv_attrs<EpiSwiGLU>()) != cudaSuccess) return e;
     if ((e = set_gemv_attrs<EpiQKV>()) != cudaSuccess) return e;
@@ -830,9 +831,36 @@ static GemvIn gemv_in(const Plan &p, const Bufs &b, const uint16_t *W, int K, in
     return g;
 }
 
+// Decode-step GEMVs in launch order: per layer QKV, O, gate/up, down; then the LM head.
+enum GemvId : int { G_QKV = 0, G_O = 1, G_GU = 2, G_DOWN = 3, G_LM = 4 };
+
+static void set_next(const Plan &p, const Bufs &b, GemvIn &g, int layer, int id) {
+    if (id == G_LM) {
+        layer = 0;
+        id = G_QKV;        // the next step starts with layer 0
+    } else if (id == G_DOWN) {
+        if (++layer == p.L) id = G_LM;
+        else id = G_QKV;
+    } else {
+        ++id;
+    }
+    if (id == G_LM) {
+        g.next_W = b.W + p.w_lm; g.next_K = p.H; g.next_n_units = p.V; g.next_rpu = 1;
+        return;
+    }
+    const LayerOffsets &lo = p.layer[layer];
+    switch (id) {
+        case G_QKV: g.next_W = b.W + lo.wqkv; g.next_K = p.H; g.next_n_units = p.nqkv / 2; g.next_rpu = 2; break;
+        case G_O: g.next_W = b.W + lo.wo; g.next_K = p.qdim; g.next_n_units = p.H; g.next_rpu = 1; break;
+        case G_GU: g.next_W = b.W + lo.wgu; g.next_K = p.H; g.next_n_units = p.F; g.next_rpu = 2; break;
+        default: g.next_W = b.W + lo.wd; g.next_K = p.F; g.next_n_units = p.H; g.next_rpu = 1; break;
+    }
+}
+
 cudaError_t enqueue_lm_head(const Plan &p, const Bufs &b, cudaStream_t st, bool pdl, int pos_add,
                             LaunchHook *hook) {
     GemvIn g = gemv_in(p, b, b.W + p.w_lm, p.H, p.V, 1, b.x, b.W + p.w_final_norm);
+    set_next(p, b, g, p.L - 1, G_LM);   // a decode step (layer 0) follows
     EpiArgmax e = {};
     e.logits = b.logits;
     e.partial = b.amax;
@@ -884,6 +912,7 @@ cudaError_t enqueue_decode_step(const Plan &p, const Bufs &b, cudaStream_t st, b
             g.embed = b.W + p.w_embed;
             g.x_out = b.x;
         }
+        set_next(p, b, g, l, G_QKV);
         EpiQKV eq = {};
         eq.q = b.q;
         eq.kv = kvl;
@@ -898,7 +927,8 @@ cudaError_t enqueue_decode_step(const Plan &p, const Bufs &b, cudaStream_t st, b
         eq.page_elems = p.kv_page_elems;
         if ((e = launch_gemv(p, g, eq, st, pdl && l > 0, hook, "qkv_rope_kvappend")) != cudaSuccess) return e;
         // A5: attention
-        FDArgs fa = {b.q, kvl, b.pages, b.ctrl, b.o, p.nkv, p.group, fd_wph(p.group), p.kv_page_elems, qscale};
+        FDArgs fa = {b.q, kvl, b.pages, b.ctrl, b.o, b.fd_part, p.nkv, p.group, fd_wph(p.group), p.kv_page_elems,
+                     qscale};
         if (hook) hook->before("flash_decode");
         if (p.d == 128)
             e = launch_fd<128>(p, fa, st, pdl);
@@ -908,14 +938,17 @@ cudaError_t enqueue_decode_step(const Plan &p, const Bufs &b, cudaStream_t st, b
         if (e != cudaSuccess) return e;
         // A6: O projection + residual
         g = gemv_in(p, b, b.W + lo.wo, p.qdim, p.H, 1, b.o, nullptr);
+        set_next(p, b, g, l, G_O);
         if ((e = launch_gemv(p, g, EpiResidual{b.x}, st, pdl, hook, "o_proj_residual")) != cudaSuccess)
             return e;
         // A7: RMSNorm + gate/up + SwiGLU
         g = gemv_in(p, b, b.W + lo.wgu, p.H, p.F, 2, b.x, b.W + lo.ffn_norm);
+        set_next(p, b, g, l, G_GU);
         if ((e = launch_gemv(p, g, EpiSwiGLU{b.m}, st, pdl, hook, "gate_up_swiglu")) != cudaSuccess)
             return e;
         // A8: down projection + residual
         g = gemv_in(p, b, b.W + lo.wd, p.F, p.H, 1, b.m, nullptr);
+        set_next(p, b, g, l, G_DOWN);
         if ((e = launch_gemv(p, g, EpiResidual{b.x}, st, pdl, hook, "down_residual")) != cudaSuccess)
             return e;
     }

@@ -125,6 +125,7 @@ const char *wici::make_plan(const wici_config *cfg, int num_sms, Plan *p) {
     P.ws_m = ws(F * 4);
     P.ws_logits = ws(V * 4);
     P.ws_amax = ws((size_t)P.num_sms * sizeof(int2));
+    P.ws_fd_part = ws(fd_part_floats(P.nkv, P.group, P.d, P.max_pages) * sizeof(float));
     P.ws_rope = ws((size_t)c.max_tokens * (P.d / 2) * sizeof(float2));
     P.ws_pages = ws((size_t)P.max_pages * 4);
     P.ws_tok = ws(T * 4);
@@ -152,6 +153,7 @@ static Bufs make_bufs(const Plan &p, void *W, void *KV, void *WS) {
     b.m = (float *)(ws + p.ws_m);
     b.logits = (float *)(ws + p.ws_logits);
     b.amax = (int2 *)(ws + p.ws_amax);
+    b.fd_part = (float *)(ws + p.ws_fd_part);
     b.rope = (float2 *)(ws + p.ws_rope);
     b.pages = (int *)(ws + p.ws_pages);
     b.tok = (int *)(ws + p.ws_tok);

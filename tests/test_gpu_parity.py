@@ -71,6 +71,13 @@ def test_agentic_turns_two_layers_chunked():
     _workload(cfg, max_chunk=128)
 
 
+def test_agentic_long_context_two_layers():
+    # past 2048 cached tokens the flash-decode splits hold more pages than its ring
+    cfg = gen.LLAMA_8B_AGENTIC.with_(name="agentic-long-2l", n_layers=2, prompt_len=1100, decode_steps=4, turns=2,
+                                     prompt_seeds=(1, 2))
+    _workload(cfg, max_chunk=512)
+
+
 def _tiny_model(max_tokens=64, **kw):
     cfg = gen.TINY
     return cfg, WiciModel(cfg, max_tokens=max_tokens, **kw).load(weights(cfg))
