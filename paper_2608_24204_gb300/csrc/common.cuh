@@ -13,6 +13,7 @@ enum CtrlSlot : int {
     CTRL_TOKEN = 1,      // input token of the next step / last greedy token
     CTRL_ERR = 2,        // nonzero: a bounded wait gave up (site id)
     CTRL_LM_TICKET = 3,  // last-CTA ticket of the LM-head argmax
+    CTRL_GRID_BAR = 4,   // arrival counter of the decode-step kernel's grid barriers
     CTRL_ATTN_TICKET0 = 16,  // per KV head tickets of the flash-decode combine
     CTRL_WORDS = 128,
 };

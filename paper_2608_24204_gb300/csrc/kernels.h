@@ -68,6 +68,9 @@ cudaError_t enqueue_lm_head_argmax_raw(const uint16_t *W, const uint16_t *gain, 
                                        float eps, float *logits, int *ctrl, int2 *partials, int *hist, int grid,
                                        cudaStream_t st);
 
+// True when the decode step runs as one persistent kernel for this plan.
+bool decode_is_persistent(const Plan &p);
+
 // Whole decode step for the token in ctrl[CTRL_TOKEN] at position ctrl[CTRL_POS]:
 // 5 launches per layer + the LM head.  `pdl` enables programmatic dependent launch.
 cudaError_t enqueue_decode_step(const Plan &p, const Bufs &b, cudaStream_t st, bool pdl,

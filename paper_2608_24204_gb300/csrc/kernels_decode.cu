@@ -43,7 +43,8 @@ struct GemvIn {
 struct EpiResidual {  // x[u] += W x_in   (O projection, down projection)
     float *x;
     static constexpr bool kArgmax = false;
-    __device__ void unit(int u, const float *v) { x[u] += v[0]; }
+    // x is read at L2 (.cg): inside the persistent decode kernel other SMs write it
+    __device__ void unit(int u, const float *v) { x[u] = __ldcg(x + u) + v[0]; }
 };
 
 struct EpiSwiGLU {    // rows (2u, 2u+1) are (gate_u, up_u): m[u] = silu(g) * u
@@ -151,6 +152,19 @@ constexpr int kGemvConsumers = 256;
 constexpr int kGemvWarps = 8;
 
 __device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
+// consumer barrier that also returns the OR of every consumer thread's flag, so
+// all of them take the same branch afterwards
+__device__ __forceinline__ bool consumer_sync_or(bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 q, %1, 0;\n\t"
+        "bar.red.or.pred p, 1, 256, q;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)v)
+        : "memory");
+    return r != 0;
+}
 
 __device__ __forceinline__ uint4 lds128(uint32_t addr) {
     uint4 r;
@@ -652,18 +666,21 @@ __global__ void __launch_bounds__(32 * (kFdMaxQueryWarps + 1)) flash_decode_kern
         else
             *reinterpret_cast<float2 *>(mine + lane * 2) = make_float2(acc[0], acc[1]);
         if (lane == 0) *reinterpret_cast<float2 *>(mine + D) = make_float2(m, l);
-        __threadfence();
     }
+    // the CTA barrier orders every warp's stores before thread 0's fence, which
+    // publishes them at GPU scope ahead of the ticket (and, for the last CTA, orders
+    // the other splits' stores before the loads below)
     asm volatile("bar.sync 1, %0;" ::"r"(32 * nq) : "memory");
     if (threadIdx.x == 0) {
+        __threadfence();
         const int t = atomicAdd(a.ctrl + CTRL_ATTN_TICKET0 + g, 1);
         s_last = (t == splits - 1);
+        if (s_last) __threadfence();
     }
     asm volatile("bar.sync 1, %0;" ::"r"(32 * nq) : "memory");
     if (!s_last || set != 0) return;
 
     // ------------------------------------------- last CTA of head g: combine
-    __threadfence();
     const float *base = a.part + ((size_t)g * gridDim.x * a.group + j) * STRIDE;
     const size_t sstride = (size_t)a.group * STRIDE;     // floats between splits of one head
     float2 ml = make_float2(-INFINITY, 0.f);
@@ -705,6 +722,625 @@ __global__ void __launch_bounds__(32 * (kFdMaxQueryWarps + 1)) flash_decode_kern
     if (j == 0 && lane == 0) a.ctrl[CTRL_ATTN_TICKET0 + g] = 0;   // ready for the next layer
 }
 
+// ======================================================= persistent decode ====
+// The whole decode step (Sec. 5.1: one forward pass per generated token) as one
+// cooperative kernel, one CTA per SM.  Weight streaming does not depend on the
+// data, so the producer warp walks the step's weights (per layer: this CTA's
+// rows of Wqkv, its KV pages, its rows of Wo, Wg|Wu and Wd; then the LM head)
+// through one TMA ring without ever waiting on a data dependency, only on free
+// ring slots.  The eight consumer warps run the phases in order and meet at a
+// grid barrier wherever a phase needs every CTA's output (the normalised
+// residual, the attention output, the SwiGLU vector).  While the consumers wait
+// at a barrier the ring keeps filling, so the HBM stays busy across the phase
+// boundaries that separate kernels in the multi-launch path.
+//
+// Data written by one CTA and read by another inside the launch (x, q, o, m,
+// the attention split states, this step's K/V row) is read at L2 (.cg loads),
+// never from a possibly stale L1 line.
+constexpr int kMegaSlots = 6;
+constexpr uint32_t kMegaSlotBytes = 32768;
+constexpr size_t kMegaSmem = kGemvRedBytes + (size_t)kMegaSlots * kMegaSlotBytes;
+
+enum : int { SITE_MEGA_EMPTY = 51, SITE_MEGA_FULL = 52, SITE_MEGA_DRAIN = 53, SITE_MEGA_GRID = 54 };
+
+template <int NCH_, int RPS_, bool FULL_>
+struct GShape {
+    static constexpr int NCH = NCH_, RPS = RPS_;
+    static constexpr bool FULL = FULL_;
+};
+
+struct MegaArgs {
+    const uint16_t *W;          // weight arena
+    size_t lstride;             // elements between the same tensor of consecutive layers
+    LayerOffsets l0;            // layer 0 offsets
+    size_t w_embed, w_final_norm, w_lm;
+    uint16_t *KV;
+    size_t kv_layer_elems, page_elems;
+    int *ctrl, *hist;
+    float *x, *q, *o, *m, *logits;
+    int2 *amax;
+    const float2 *rope;
+    const int *pages;
+    float *part;                // attention split states [nkv][splits][group][d + 4]
+    int L, H, F, V, nqkv, qdim, kvdim, d, nkv, group, wph, splits;
+    int bias;
+    float eps, qscale;
+};
+
+struct MegaRing {
+    uint32_t full0, empty0, data0;   // shared-memory addresses
+    const uint8_t *ring;             // generic pointer to slot 0
+    int n;   // slots issued (producer) or consumed (consumer) so far
+    int *abort;                      // shared flag: a consumer wait gave up
+};
+
+__device__ __forceinline__ int mega_u0(int n_units) {
+    return (int)(((long long)blockIdx.x * n_units) / gridDim.x);
+}
+
+// ----------------------------------------------------------- producer side --
+__device__ bool mp_rows(MegaRing &R, const uint16_t *W, int K, int n_units, int rpu, int RPS, int *err,
+                        uint64_t pol) {
+    const int u0 = mega_u0(n_units);
+    const int u1 = (int)(((long long)(blockIdx.x + 1) * n_units) / gridDim.x);
+    const int total_rows = (u1 - u0) * rpu;
+    const int nst = (total_rows + RPS - 1) / RPS;
+    const uint16_t *src = W + (size_t)u0 * rpu * K;
+    for (int s = 0; s < nst; ++s) {
+        const int slot = R.n % kMegaSlots;
+        if (R.n >= kMegaSlots &&
+            !mbar_wait(R.empty0 + 8 * slot, ((R.n / kMegaSlots) + 1) & 1, err, SITE_MEGA_EMPTY))
+            return false;
+        const int rows = min(RPS, total_rows - s * RPS);
+        const uint32_t bytes = (uint32_t)rows * (uint32_t)K * 2u;
+        mbar_arrive_expect_tx(R.full0 + 8 * slot, bytes);
+        bulk_g2s(R.data0 + slot * kMegaSlotBytes, src + (size_t)s * RPS * K, bytes, R.full0 + 8 * slot, pol);
+        ++R.n;
+    }
+    return true;
+}
+
+// the pages of this CTA's attention split (its K and V blocks), one page per slot
+struct MegaSplit {
+    int g, r, p0, n, npages, splits;
+    bool active;
+};
+
+__device__ __forceinline__ MegaSplit mega_split(const MegaArgs &a, int len) {
+    MegaSplit sp;
+    const int unit = blockIdx.x;
+    sp.npages = (len + kPage - 1) / kPage;
+    const int pps = (sp.npages + a.splits - 1) / a.splits;
+    sp.splits = (sp.npages + pps - 1) / pps;
+    sp.g = unit / a.splits;
+    sp.r = unit % a.splits;
+    sp.active = unit < a.nkv * a.splits && sp.r < sp.splits;
+    sp.p0 = sp.r * pps;
+    sp.n = sp.active ? min(sp.npages, sp.p0 + pps) - sp.p0 : 0;
+    return sp;
+}
+
+template <int D>
+__device__ bool mp_pages(MegaRing &R, const MegaArgs &a, const uint16_t *kvl, const MegaSplit &sp, int *err) {
+    constexpr uint32_t BLK = kPage * D * 2;
+    for (int i = 0; i < sp.n; ++i) {
+        const int slot = R.n % kMegaSlots;
+        if (R.n >= kMegaSlots &&
+            !mbar_wait(R.empty0 + 8 * slot, ((R.n / kMegaSlots) + 1) & 1, err, SITE_MEGA_EMPTY))
+            return false;
+        const int page = a.pages[sp.p0 + i];
+        const uint16_t *Kb = kvl + (size_t)page * a.page_elems + (size_t)sp.g * kPage * D;
+        const uint16_t *Vb = Kb + (size_t)a.nkv * kPage * D;
+        mbar_arrive_expect_tx(R.full0 + 8 * slot, 2 * BLK);
+        bulk_g2s(R.data0 + slot * kMegaSlotBytes, Kb, BLK, R.full0 + 8 * slot);
+        bulk_g2s(R.data0 + slot * kMegaSlotBytes + BLK, Vb, BLK, R.full0 + 8 * slot);
+        ++R.n;
+    }
+    return true;
+}
+
+// ----------------------------------------------------------- consumer side --
+// consumers only (8 warps): bar.sync 1, 256 is consumer_sync()
+
+// Grid barrier number k (1-based): every CTA's consumer writes so far are visible
+// to every CTA afterwards.  Gives up after kWaitLimitNs, or at once when another
+// CTA has recorded an error.
+__device__ bool mega_grid_sync(int *ctrl, int k, int *s_flag) {
+    consumer_sync();
+    if (threadIdx.x == 0) {
+        int *ctr = ctrl + CTRL_GRID_BAR;
+        const int target = k * (int)gridDim.x;
+        __threadfence();
+        atomicAdd(ctr, 1);
+        bool ok = false;
+        const uint64_t t0 = globaltimer_ns();
+        for (uint32_t it = 0; it < 0x7FFFFFFFu; ++it) {
+            int v;
+            asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+            if (v >= target) {
+                ok = true;
+                break;
+            }
+            if (*reinterpret_cast<volatile int *>(ctrl + CTRL_ERR) != 0) break;
+            if ((it & 15u) == 15u && globaltimer_ns() - t0 > kWaitLimitNs) {
+                atomicCAS(ctrl + CTRL_ERR, 0, SITE_MEGA_GRID);
+                break;
+            }
+            __nanosleep(20);
+        }
+        __threadfence();
+        *s_flag = ok ? 1 : 0;
+    }
+    consumer_sync();
+    return *s_flag != 0;
+}
+
+// One GEMV phase of the consumers: the rows of units [u0, u1) of a K-column matrix
+// against `in` (RMSNorm'd with `gain` when given; layer 0 reads embed[token]).
+template <class SH, class Epi>
+__device__ bool mc_gemv(MegaRing &R, float *red, int K, int n_units, int rpu, const float *in,
+                        const uint16_t *gain, const uint16_t *embed, float *x_out, float eps, int *ctrl, Epi &epi,
+                        float *s_part) {
+    constexpr int NCH = SH::NCH, RPS = SH::RPS;
+    constexpr bool FULL = SH::FULL;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int u0 = mega_u0(n_units);
+    const int u1 = (int)(((long long)(blockIdx.x + 1) * n_units) / gridDim.x);
+    const int total_rows = (u1 - u0) * rpu;
+    const int nst = (total_rows + RPS - 1) / RPS;
+    int *err = ctrl + CTRL_ERR;
+    const int nchunks = K >> 3;
+    float h[NCH][8];
+    float ss = 0.f;
+    const int tok = embed ? ctrl[CTRL_TOKEN] : 0;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+        const int c = tid + kGemvConsumers * j;
+        if (FULL || c < nchunks) {
+            if (embed) {
+                const uint4 w = *reinterpret_cast<const uint4 *>(embed + (size_t)tok * K + c * 8);
+                h[j][0] = bf16lo(w.x); h[j][1] = bf16hi(w.x); h[j][2] = bf16lo(w.y); h[j][3] = bf16hi(w.y);
+                h[j][4] = bf16lo(w.z); h[j][5] = bf16hi(w.z); h[j][6] = bf16lo(w.w); h[j][7] = bf16hi(w.w);
+                if (blockIdx.x == 0) {
+                    float4 *dst = reinterpret_cast<float4 *>(x_out + c * 8);
+                    dst[0] = make_float4(h[j][0], h[j][1], h[j][2], h[j][3]);
+                    dst[1] = make_float4(h[j][4], h[j][5], h[j][6], h[j][7]);
+                }
+            } else {
+                const float4 a = __ldcg(reinterpret_cast<const float4 *>(in + c * 8));
+                const float4 b = __ldcg(reinterpret_cast<const float4 *>(in + c * 8 + 4));
+                h[j][0] = a.x; h[j][1] = a.y; h[j][2] = a.z; h[j][3] = a.w;
+                h[j][4] = b.x; h[j][5] = b.y; h[j][6] = b.z; h[j][7] = b.w;
+            }
+#pragma unroll
+            for (int e = 0; e < 8; ++e) ss = fmaf(h[j][e], h[j][e], ss);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) h[j][e] = 0.f;
+        }
+    }
+    if (gain) {
+        ss = warp_sum(ss);
+        if (lane == 0) s_part[warp] = ss;
+        consumer_sync();
+        float tot = 0.f;
+#pragma unroll
+        for (int w = 0; w < kGemvWarps; ++w) tot += s_part[w];
+        const float rinv = 1.0f / sqrtf(tot / (float)K + eps);
+#pragma unroll
+        for (int j = 0; j < NCH; ++j) {
+            const int c = tid + kGemvConsumers * j;
+            if (FULL || c < nchunks) {
+                const uint4 gw = *reinterpret_cast<const uint4 *>(gain + c * 8);
+                const float gg[8] = {bf16lo(gw.x), bf16hi(gw.x), bf16lo(gw.y), bf16hi(gw.y),
+                                     bf16lo(gw.z), bf16hi(gw.z), bf16lo(gw.w), bf16hi(gw.w)};
+#pragma unroll
+                for (int e = 0; e < 8; ++e) h[j][e] = h[j][e] * rinv * gg[e];
+            }
+        }
+    }
+
+    const uint32_t row_bytes = (uint32_t)K * 2u;
+    const bool tail_ok = FULL || tid + kGemvConsumers * (NCH - 1) < nchunks;
+    int buf = 0, brow = 0, bunit0 = 0;
+    bool ok = true;
+    for (int s = 0; s < nst; ++s) {
+        const int slot = R.n % kMegaSlots;
+        const int rows = min(RPS, total_rows - s * RPS);
+        // after a wait gives up every thread still reaches the same barriers; they
+        // leave together at the next flush
+        ok = ok && !*reinterpret_cast<volatile int *>(R.abort) &&
+             mbar_wait(R.full0 + 8 * slot, (R.n / kMegaSlots) & 1, err, SITE_MEGA_FULL);
+        if (!ok) *R.abort = 1;
+        float acc[RPS];
+#pragma unroll
+        for (int r = 0; r < RPS; ++r) acc[r] = 0.f;
+        const uint32_t sb = R.data0 + (uint32_t)slot * kMegaSlotBytes + (uint32_t)tid * 16u;
+        if (!ok) {
+        } else if (rows == RPS) {
+#pragma unroll
+            for (int r = 0; r < RPS; ++r)
+#pragma unroll
+                for (int j = 0; j < NCH; ++j)
+                    if (j < NCH - 1 || tail_ok)
+                        acc[r] = dot8(lds128(sb + r * row_bytes + j * kGemvConsumers * 16), h[j], acc[r]);
+        } else {
+#pragma unroll
+            for (int r = 0; r < RPS; ++r)
+                if (r < rows)
+#pragma unroll
+                    for (int j = 0; j < NCH; ++j)
+                        if (j < NCH - 1 || tail_ok)
+                            acc[r] = dot8(lds128(sb + r * row_bytes + j * kGemvConsumers * 16), h[j], acc[r]);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(R.empty0 + 8 * slot);
+        ++R.n;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+            for (int r = 0; r < RPS; ++r) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
+        if (lane == 0) {
+            float *rb = red + (size_t)(buf * kGemvWarps + warp) * kRedRows + brow;
+#pragma unroll
+            for (int r = 0; r < RPS; ++r)
+                if (r < rows) rb[r] = acc[r];
+        }
+        brow += rows;
+        if (s == nst - 1 || brow + RPS > kRedRows) {
+            if (consumer_sync_or(!ok)) return false;
+            const int bunits = brow / rpu;
+            for (int t = tid; t < bunits; t += kGemvConsumers) {
+                float v[2];
+                for (int j = 0; j < rpu; ++j) {
+                    float sum = 0.f;
+#pragma unroll
+                    for (int w = 0; w < kGemvWarps; ++w)
+                        sum += red[(size_t)(buf * kGemvWarps + w) * kRedRows + t * rpu + j];
+                    v[j] = sum;
+                }
+                epi.unit(u0 + bunit0 + t, v);
+            }
+            bunit0 += bunits;
+            brow = 0;
+            buf ^= 1;
+        }
+    }
+    return true;
+}
+
+// Attention of the current token for this CTA's split (KV head g, pages
+// [p0, p0 + n)), then the split state to global memory and the ticket; the last
+// split of head g combines the states in split order into o.  Warp (j, set) with
+// j = warp % group handles query head g*group + j on pages i = set (mod wph);
+// warps beyond group * wph only keep the ring in step.
+template <int D>
+__device__ bool mc_attn(MegaRing &R, const MegaArgs &a, const uint16_t *kvl, const MegaSplit &sp, int len,
+                        float (*s_state)[D + 4], int *s_last) {
+    constexpr int EPL = D / 32;
+    constexpr uint32_t BLK = kPage * D * 2;
+    constexpr int STRIDE = D + 4;
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nq = a.group * a.wph;
+    int *err = a.ctrl + CTRL_ERR;
+    if (!sp.active) return true;
+    const int j = w % a.group, set = w / a.group;
+    const bool qwarp = w < nq;
+    const int head = sp.g * a.group + j;
+    float qv[EPL], acc[EPL];
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
+    if (qwarp) {
+        if constexpr (EPL == 4) {
+            const float4 q4 = __ldcg(reinterpret_cast<const float4 *>(a.q + head * D + lane * 4));
+            qv[0] = q4.x * a.qscale; qv[1] = q4.y * a.qscale; qv[2] = q4.z * a.qscale; qv[3] = q4.w * a.qscale;
+        } else {
+            const float2 q2 = __ldcg(reinterpret_cast<const float2 *>(a.q + head * D + lane * 2));
+            qv[0] = q2.x * a.qscale; qv[1] = q2.y * a.qscale;
+        }
+    }
+    // this step's K/V row was written by another CTA during the QKV phase, possibly
+    // after the producer copied its page: it is read from L2 instead of the ring
+    const int cur_slot = (len - 1) % kPage;
+    uint32_t kcur[EPL / 2], vcur[EPL / 2];
+    if (qwarp && sp.p0 + sp.n == sp.npages) {
+        const int page = a.pages[sp.npages - 1];
+        const uint16_t *kr = kvl + (size_t)page * a.page_elems + ((size_t)sp.g * kPage + cur_slot) * D + lane * EPL;
+        const uint16_t *vr = kr + (size_t)a.nkv * kPage * D;
+        if constexpr (EPL == 4) {
+            const uint2 k2 = __ldcg(reinterpret_cast<const uint2 *>(kr));
+            const uint2 v2 = __ldcg(reinterpret_cast<const uint2 *>(vr));
+            kcur[0] = k2.x; kcur[1] = k2.y; vcur[0] = v2.x; vcur[1] = v2.y;
+        } else {
+            kcur[0] = __ldcg(reinterpret_cast<const unsigned int *>(kr));
+            vcur[0] = __ldcg(reinterpret_cast<const unsigned int *>(vr));
+        }
+    }
+    float m = -INFINITY, l = 0.f;
+    const int key = lane >> 1;
+    bool ok = true;
+    for (int i = 0; i < sp.n; ++i) {
+        const int slot = R.n % kMegaSlots;
+        ok = ok && !*reinterpret_cast<volatile int *>(R.abort) &&
+             mbar_wait(R.full0 + 8 * slot, (R.n / kMegaSlots) & 1, err, SITE_MEGA_FULL);
+        if (!ok) *R.abort = 1;
+        if (ok && qwarp && (i % a.wph) == set) {
+            const uint8_t *Ks = R.ring + (size_t)slot * kMegaSlotBytes;
+            const uint8_t *Vs = Ks + BLK;
+            const int ntok = min(kPage, len - (sp.p0 + i) * kPage);
+            const int ct = (sp.p0 + i == sp.npages - 1) ? cur_slot : -1;
+            float sc[kPage];
+#pragma unroll
+            for (int t = 0; t < kPage; ++t) {
+                const uint8_t *kr = Ks + (t * D + lane * EPL) * 2;
+                if constexpr (EPL == 4) {
+                    uint2 kw = *reinterpret_cast<const uint2 *>(kr);
+                    if (t == ct) kw = make_uint2(kcur[0], kcur[1]);
+                    sc[t] = qv[0] * bf16lo(kw.x) + qv[1] * bf16hi(kw.x) + qv[2] * bf16lo(kw.y) +
+                            qv[3] * bf16hi(kw.y);
+                } else {
+                    uint32_t kw = *reinterpret_cast<const uint32_t *>(kr);
+                    if (t == ct) kw = kcur[0];
+                    sc[t] = qv[0] * bf16lo(kw) + qv[1] * bf16hi(kw);
+                }
+            }
+#pragma unroll
+            for (int o = 16, cnt = kPage; o > 0; o >>= 1) {
+                if (cnt > 1) {
+                    const bool up = (lane & o) != 0;
+#pragma unroll
+                    for (int t = 0; t < cnt / 2; ++t) {
+                        const float send = up ? sc[t] : sc[t + cnt / 2];
+                        const float keep = up ? sc[t + cnt / 2] : sc[t];
+                        sc[t] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+                    }
+                    cnt >>= 1;
+                } else {
+                    sc[0] += __shfl_xor_sync(0xffffffffu, sc[0], o);
+                }
+            }
+            const float my = key < ntok ? sc[0] : -INFINITY;
+            const float mx = fmaxf(m, warp_max(my));
+            const float corr = exp2f(m - mx);
+            const float pme = exp2f(my - mx);
+            l = l * corr + pme;
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) acc[e] *= corr;
+#pragma unroll
+            for (int t = 0; t < kPage; ++t) {
+                const bool valid = t < ntok;
+                const float pt = __shfl_sync(0xffffffffu, pme, 2 * t);
+                const uint8_t *vr = Vs + (t * D + lane * EPL) * 2;
+                if constexpr (EPL == 4) {
+                    uint2 vw = *reinterpret_cast<const uint2 *>(vr);
+                    if (t == ct) vw = make_uint2(vcur[0], vcur[1]);
+                    if (!valid) vw = make_uint2(0u, 0u);
+                    acc[0] = fmaf(pt, bf16lo(vw.x), acc[0]);
+                    acc[1] = fmaf(pt, bf16hi(vw.x), acc[1]);
+                    acc[2] = fmaf(pt, bf16lo(vw.y), acc[2]);
+                    acc[3] = fmaf(pt, bf16hi(vw.y), acc[3]);
+                } else {
+                    uint32_t vw = *reinterpret_cast<const uint32_t *>(vr);
+                    if (t == ct) vw = vcur[0];
+                    if (!valid) vw = 0u;
+                    acc[0] = fmaf(pt, bf16lo(vw), acc[0]);
+                    acc[1] = fmaf(pt, bf16hi(vw), acc[1]);
+                }
+            }
+            m = mx;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(R.empty0 + 8 * slot);
+        ++R.n;
+    }
+    if (consumer_sync_or(!ok)) return false;
+    l = warp_sum(l) * 0.5f;
+    if (a.wph > 1) {
+        if (qwarp) {
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) s_state[w][lane * EPL + e] = acc[e];
+            if (lane == 0) {
+                s_state[w][D] = m;
+                s_state[w][D + 1] = l;
+            }
+        }
+        consumer_sync();
+        if (qwarp && set == 0)
+            for (int t = 1; t < a.wph; ++t) {
+                const float *o = s_state[t * a.group + j];
+                float ob[EPL];
+#pragma unroll
+                for (int e = 0; e < EPL; ++e) ob[e] = o[lane * EPL + e];
+                fd_merge<EPL>(m, l, acc, o[D], o[D + 1], ob);
+            }
+    }
+    const bool writer = qwarp && set == 0;
+    if (writer) {
+        float *mine = a.part + ((size_t)(sp.g * a.splits + sp.r) * a.group + j) * STRIDE;
+        if constexpr (EPL == 4)
+            *reinterpret_cast<float4 *>(mine + lane * 4) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+        else
+            *reinterpret_cast<float2 *>(mine + lane * 2) = make_float2(acc[0], acc[1]);
+        if (lane == 0) *reinterpret_cast<float2 *>(mine + D) = make_float2(m, l);
+    }
+    consumer_sync();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const int t = atomicAdd(a.ctrl + CTRL_ATTN_TICKET0 + sp.g, 1);
+        *s_last = (t == sp.splits - 1);
+        if (*s_last) __threadfence();
+    }
+    consumer_sync();
+    if (!*s_last || !writer) return true;
+
+    const float *base = a.part + ((size_t)sp.g * a.splits * a.group + j) * STRIDE;
+    const size_t sstride = (size_t)a.group * STRIDE;
+    float2 ml = make_float2(-INFINITY, 0.f);
+    if (lane < sp.splits) ml = __ldcg(reinterpret_cast<const float2 *>(base + lane * sstride + D));
+    const float M = warp_max(ml.x);
+    const float f = lane < sp.splits ? exp2f(ml.x - M) : 0.f;
+    const float Lsum = warp_sum(ml.y * f);
+    float out[EPL];
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) out[e] = 0.f;
+    for (int s0 = 0; s0 < sp.splits; s0 += 8) {
+        float v[8][EPL];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int si = min(s0 + u, sp.splits - 1);
+            const float *src = base + si * sstride + lane * EPL;
+            if constexpr (EPL == 4) {
+                const float4 t4 = __ldcg(reinterpret_cast<const float4 *>(src));
+                v[u][0] = t4.x; v[u][1] = t4.y; v[u][2] = t4.z; v[u][3] = t4.w;
+            } else {
+                const float2 t2 = __ldcg(reinterpret_cast<const float2 *>(src));
+                v[u][0] = t2.x; v[u][1] = t2.y;
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const float fs = __shfl_sync(0xffffffffu, f, (s0 + u) & 31);
+            if (s0 + u < sp.splits)
+#pragma unroll
+                for (int e = 0; e < EPL; ++e) out[e] = fmaf(v[u][e], fs, out[e]);
+        }
+    }
+    const float inv = 1.0f / Lsum;
+    if constexpr (EPL == 4)
+        *reinterpret_cast<float4 *>(a.o + head * D + lane * 4) =
+            make_float4(out[0] * inv, out[1] * inv, out[2] * inv, out[3] * inv);
+    else
+        *reinterpret_cast<float2 *>(a.o + head * D + lane * 2) = make_float2(out[0] * inv, out[1] * inv);
+    if (j == 0 && lane == 0) a.ctrl[CTRL_ATTN_TICKET0 + sp.g] = 0;
+    return true;
+}
+
+template <int D, class SH, class SF>
+__global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const MegaArgs a) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    float *red = reinterpret_cast<float *>(smem);
+    __shared__ __align__(8) uint64_t bars[2 * kMegaSlots];
+    __shared__ __align__(16) float s_state[kFdMaxQueryWarps][D + 4];
+    __shared__ float s_part[kGemvWarps];
+    __shared__ float s_bv[kGemvWarps];
+    __shared__ int s_bi[kGemvWarps];
+    __shared__ int s_flag, s_last, s_abort;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    int *err = a.ctrl + CTRL_ERR;
+
+    MegaRing R;
+    R.full0 = smem_u32(bars);
+    R.empty0 = smem_u32(bars + kMegaSlots);
+    R.data0 = smem_u32(smem + kGemvRedBytes);
+    R.ring = smem + kGemvRedBytes;
+    R.n = 0;
+    R.abort = &s_abort;
+    if (tid == 0) {
+        s_abort = 0;
+        for (int s = 0; s < kMegaSlots; ++s) {
+            mbar_init(R.full0 + 8 * s, 1);
+            mbar_init(R.empty0 + 8 * s, kGemvWarps);
+        }
+        fence_barrier_init();
+    }
+    __syncthreads();
+
+    // the position only changes at the very end of the step (last LM-head CTA)
+    const int len = *reinterpret_cast<volatile int *>(a.ctrl + CTRL_POS) + 1;
+    const MegaSplit sp = mega_split(a, len);
+
+    if (warp == kGemvWarps) {  // ------------------------------------ producer
+        if (lane == 0) {
+            const uint64_t pol = l2_evict_first();
+            bool ok = true;
+            for (int l = 0; l < a.L && ok; ++l) {
+                const size_t lo = (size_t)l * a.lstride;
+                ok = mp_rows(R, a.W + a.l0.wqkv + lo, a.H, a.nqkv / 2, 2, SH::RPS, err, pol) &&
+                     mp_pages<D>(R, a, a.KV + (size_t)l * a.kv_layer_elems, sp, err) &&
+                     mp_rows(R, a.W + a.l0.wo + lo, a.qdim, a.H, 1, SH::RPS, err, pol) &&
+                     mp_rows(R, a.W + a.l0.wgu + lo, a.H, a.F, 2, SH::RPS, err, pol) &&
+                     mp_rows(R, a.W + a.l0.wd + lo, a.F, a.H, 1, SF::RPS, err, pol);
+            }
+            if (ok) mp_rows(R, a.W + a.w_lm, a.H, a.V, 1, SH::RPS, err, pol);
+            // no copy may still be landing in shared memory when the CTA exits
+            for (int s = max(0, R.n - kMegaSlots); s < R.n; ++s)
+                mbar_wait(R.full0 + 8 * (s % kMegaSlots), (s / kMegaSlots) & 1, err, SITE_MEGA_DRAIN);
+        }
+        return;
+    }
+
+    // ---------------------------------------------------------------- consumers
+    int k = 0;   // grid barriers passed
+    bool ok = true;
+    for (int l = 0; l < a.L && ok; ++l) {
+        const size_t lo = (size_t)l * a.lstride;
+        uint16_t *kvl = a.KV + (size_t)l * a.kv_layer_elems;
+        if (l > 0) ok = mega_grid_sync(a.ctrl, ++k, &s_flag);
+        if (!ok) break;
+        EpiQKV eq;
+        eq.q = a.q; eq.kv = kvl; eq.pages = a.pages; eq.rope = a.rope; eq.ctrl = a.ctrl;
+        eq.bias = a.bias ? a.W + a.l0.bqkv + lo : nullptr;
+        eq.qdim = a.qdim; eq.kvdim = a.kvdim; eq.d = a.d; eq.nkv = a.nkv; eq.page_elems = a.page_elems;
+        ok = mc_gemv<SH>(R, red, a.H, a.nqkv / 2, 2, a.x, a.W + a.l0.attn_norm + lo,
+                         l == 0 ? a.W + a.w_embed : nullptr, a.x, a.eps, a.ctrl, eq, s_part) &&
+             mega_grid_sync(a.ctrl, ++k, &s_flag) &&
+             mc_attn<D>(R, a, kvl, sp, len, s_state, &s_last) &&
+             mega_grid_sync(a.ctrl, ++k, &s_flag);
+        if (!ok) break;
+        EpiResidual er{a.x};
+        ok = mc_gemv<SH>(R, red, a.qdim, a.H, 1, a.o, nullptr, nullptr, nullptr, a.eps, a.ctrl, er, s_part) &&
+             mega_grid_sync(a.ctrl, ++k, &s_flag);
+        if (!ok) break;
+        EpiSwiGLU es{a.m};
+        ok = mc_gemv<SH>(R, red, a.H, a.F, 2, a.x, a.W + a.l0.ffn_norm + lo, nullptr, nullptr, a.eps, a.ctrl, es,
+                         s_part) &&
+             mega_grid_sync(a.ctrl, ++k, &s_flag);
+        if (!ok) break;
+        ok = mc_gemv<SF>(R, red, a.F, a.H, 1, a.m, nullptr, nullptr, nullptr, a.eps, a.ctrl, er, s_part);
+    }
+    if (ok) ok = mega_grid_sync(a.ctrl, ++k, &s_flag);
+    if (!ok) return;
+    EpiArgmax ea;
+    ea.logits = a.logits; ea.partial = a.amax; ea.ctrl = a.ctrl; ea.hist = a.hist; ea.pos_add = 1;
+    ea.best = -INFINITY; ea.bidx = 0x7fffffff;
+    if (!mc_gemv<SH>(R, red, a.H, a.V, 1, a.x, a.W + a.w_final_norm, nullptr, nullptr, a.eps, a.ctrl, ea, s_part))
+        return;
+    // CTA argmax, then the last CTA reduces every CTA's result in index order
+    float bv = ea.best;
+    int bi = ea.bidx;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        if (better(ov, oi, bv, bi)) { bv = ov; bi = oi; }
+    }
+    if (lane == 0) { s_bv[warp] = bv; s_bi[warp] = bi; }
+    consumer_sync();
+    if (tid == 0) {
+        for (int w = 1; w < kGemvWarps; ++w)
+            if (better(s_bv[w], s_bi[w], bv, bi)) { bv = s_bv[w]; bi = s_bi[w]; }
+        a.amax[blockIdx.x] = make_int2(__float_as_int(bv), bi);
+        __threadfence();
+        const int t = atomicAdd(a.ctrl + CTRL_LM_TICKET, 1);
+        if (t == (int)gridDim.x - 1) {
+            __threadfence();
+            float fv = -INFINITY;
+            int fi = 0x7fffffff;
+            for (int c = 0; c < (int)gridDim.x; ++c) {
+                const int2 pr = __ldcg(a.amax + c);
+                const float pv = __int_as_float(pr.x);
+                if (better(pv, pr.y, fv, fi)) { fv = pv; fi = pr.y; }
+            }
+            if (fi == 0x7fffffff) fi = 0;
+            const int np = a.ctrl[CTRL_POS] + 1;
+            a.ctrl[CTRL_TOKEN] = fi;
+            a.ctrl[CTRL_POS] = np;
+            a.hist[np] = fi;
+            a.ctrl[CTRL_LM_TICKET] = 0;
+        }
+    }
+}
+
 // ------------------------------------------------------------ probe kernel ----
 __global__ void bounded_wait_probe_kernel(int *err, long long limit_ns) {
     __shared__ __align__(8) uint64_t bar;
@@ -743,7 +1379,8 @@ int fd_splits(int max_pages) {
 }
 
 size_t fd_part_floats(int nkv, int group, int d, int max_pages) {
-    return (size_t)nkv * fd_splits(max_pages) * group * (d + 4);
+    (void)max_pages;   // room for the largest split count of either decode path
+    return (size_t)nkv * kFdMaxSplits * group * (d + 4);
 }
 
 template <int D>
@@ -784,8 +1421,28 @@ static cudaError_t set_gemv_attrs() {
     return cudaSuccess;
 }
 
+// The instantiated shapes: (head dim, GEMV shape of K = hidden, GEMV shape of K = ffn)
+using MegaH4096 = GShape<2, 4, true>;     // Llama-3-8B widths: hidden 4096, ffn 14336
+using MegaF14336 = GShape<7, 1, true>;
+using MegaH2048 = GShape<1, 8, true>;     // Llama-3.2-1B widths: hidden 2048, ffn 8192
+using MegaF8192 = GShape<4, 2, true>;
+using MegaH5120 = GShape<3, 2, false>;    // Qwen2.5-14B widths: hidden 5120, ffn 13824
+using MegaF13824 = GShape<7, 1, false>;
+using MegaSmall = GShape<1, 8, false>;    // hidden and ffn below 2048 (e.g. 256 / 688)
+#define WICI_MEGA_SHAPES(X)            \
+    X(128, MegaH4096, MegaF14336)      \
+    X(64, MegaH2048, MegaF8192)        \
+    X(128, MegaH5120, MegaF13824)      \
+    X(64, MegaSmall, MegaSmall)
+
 cudaError_t setup_kernels() {
     cudaError_t e;
+#define WICI_MEGA_ATTR(DD, SH, SF)                                                                  \
+    if ((e = cudaFuncSetAttribute(decode_step_kernel<DD, SH, SF>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
+                                  (int)kMegaSmem)) != cudaSuccess)                                    \
+        return e;
+    WICI_MEGA_SHAPES(WICI_MEGA_ATTR)
+#undef WICI_MEGA_ATTR
     if ((e = set_gemv_attrs<EpiResidual>()) != cudaSuccess) return e;
     if ((e = set_gemv_attrs<EpiSwiGLU>()) != cudaSuccess) return e;
     if ((e = set_gemv_attrs<EpiQKV>()) != cudaSuccess) return e;
@@ -899,8 +1556,92 @@ cudaError_t enqueue_lm_head_argmax_raw(const uint16_t *W, const uint16_t *gain, 
                   gemv_smem_bytes(g.stages, g.slot_bytes), st, false, g, e);
 }
 
+
+// ------------------------------------------------------- persistent decode: host
+typedef cudaError_t (*MegaLaunch)(const MegaArgs &, int grid, cudaStream_t);
+
+template <int D, class SH, class SF>
+static cudaError_t launch_mega(const MegaArgs &a, int grid, cudaStream_t st) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kGemvThreads);
+    cfg.dynamicSmemBytes = kMegaSmem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;   // every CTA resident: the grid barriers need it
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, decode_step_kernel<D, SH, SF>, a);
+}
+
+template <class S>
+static bool shape_is(int K) {
+    return gemv_nch(K) == S::NCH && gemv_rps(K) == S::RPS && ((K / 8) == S::NCH * kGemvConsumers) == S::FULL;
+}
+
+static MegaLaunch mega_launcher(const Plan &p) {
+    if (p.qdim != p.H || p.nkv > 64) return nullptr;
+    // every layer's tensors must sit at one fixed stride
+    if (p.L > 1) {
+        const size_t st = p.layer[1].wqkv - p.layer[0].wqkv;
+        for (int l = 0; l < p.L; ++l) {
+            const LayerOffsets &a = p.layer[l], &b = p.layer[0];
+            const size_t o = st * (size_t)l;
+            if (a.attn_norm != b.attn_norm + o || a.wqkv != b.wqkv + o || a.wo != b.wo + o ||
+                a.ffn_norm != b.ffn_norm + o || a.wgu != b.wgu + o || a.wd != b.wd + o ||
+                (p.cfg.qkv_bias && a.bqkv != b.bqkv + o))
+                return nullptr;
+        }
+    }
+#define WICI_MEGA_PICK(DD, SH, SF) \
+    if (p.d == DD && shape_is<SH>(p.H) && shape_is<SF>(p.F)) return launch_mega<DD, SH, SF>;
+    WICI_MEGA_SHAPES(WICI_MEGA_PICK)
+#undef WICI_MEGA_PICK
+    return nullptr;
+}
+
+bool decode_is_persistent(const Plan &p) { return mega_launcher(p) != nullptr; }
+
+static cudaError_t enqueue_mega(const Plan &p, const Bufs &b, cudaStream_t st, MegaLaunch fn) {
+    MegaArgs a = {};
+    a.W = b.W;
+    a.lstride = p.L > 1 ? p.layer[1].wqkv - p.layer[0].wqkv : 0;
+    a.l0 = p.layer[0];
+    a.w_embed = p.w_embed;
+    a.w_final_norm = p.w_final_norm;
+    a.w_lm = p.w_lm;
+    a.KV = b.KV;
+    a.kv_layer_elems = p.kv_layer_elems;
+    a.page_elems = p.kv_page_elems;
+    a.ctrl = b.ctrl;
+    a.hist = b.hist;
+    a.x = b.x; a.q = b.q; a.o = b.o; a.m = b.m; a.logits = b.logits;
+    a.amax = b.amax;
+    a.rope = b.rope;
+    a.pages = b.pages;
+    a.part = b.fd_part;
+    a.L = p.L; a.H = p.H; a.F = p.F; a.V = p.V;
+    a.nqkv = p.nqkv; a.qdim = p.qdim; a.kvdim = p.kvdim; a.d = p.d; a.nkv = p.nkv; a.group = p.group;
+    a.wph = fd_wph(p.group);
+    const int grid = p.num_sms;
+    a.splits = grid / p.nkv < kFdMaxSplits ? grid / p.nkv : kFdMaxSplits;
+    a.bias = p.cfg.qkv_bias;
+    a.eps = p.cfg.rms_eps;
+    a.qscale = 1.4426950408889634f / sqrtf((float)p.d);
+    cudaError_t e = cudaMemsetAsync(b.ctrl + CTRL_GRID_BAR, 0, sizeof(int), st);
+    if (e != cudaSuccess) return e;
+    return fn(a, grid, st);
+}
+
 cudaError_t enqueue_decode_step(const Plan &p, const Bufs &b, cudaStream_t st, bool pdl,
                                 LaunchHook *hook) {
+    if (MegaLaunch fn = mega_launcher(p)) {
+        if (hook) hook->before("decode_step");
+        cudaError_t e = enqueue_mega(p, b, st, fn);
+        if (hook) hook->after("decode_step");
+        return e;
+    }
     cudaError_t e;
     const float qscale = 1.4426950408889634f / sqrtf((float)p.d);
     for (int l = 0; l < p.L; ++l) {

@@ -190,3 +190,10 @@ def test_device_weights_load_like_host_weights():
     assert np.array_equal(la, lb)
     a.close()
     b.close()
+
+
+def test_multi_launch_decode_path_when_query_width_differs_from_hidden():
+    # 8 query heads x 64 = 512 != hidden 256: the decode step runs as one launch per
+    # layer operation (QKV, attention, O, gate/up, down) instead of the persistent kernel
+    cfg = gen.TINY.with_(name="tiny-wideq", n_q_heads=8, decode_steps=6)
+    _workload(cfg)
