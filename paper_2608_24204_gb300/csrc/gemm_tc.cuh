@@ -3,7 +3,7 @@
 //   C[T][N] = (A_0 + A_1 + A_2)[T][K] . W[N][K]^T,  fp32 accumulation in TMEM
 //
 // A is an fp32 activation carried as kTerms = 3 bf16 terms (split_bf16x3); W is
-// bf16 and exact.  The three products accumulate into one 128x128 fp32
+// bf16 and exact.  The three products accumulate into one fp32 TMEM
 // accumulator, so the activations keep fp32 precision on bf16 MMAs (the bf16x3
 // scheme of Henry, Tang & Heinecke, ARITH 2019, applied to one operand).
 //
@@ -15,13 +15,16 @@
 // warps fold each finished group into fp32 registers (round-to-nearest adds)
 // while the next group accumulates into the other buffer.
 //
-// One CTA computes one 128x128 output tile with three warp roles:
+// Persistent: one CTA per SM walks the output tiles (M tiles fastest, so the
+// CTAs that run together share a weight tile through L2) with three warp roles:
 //   warp 0      TMA producer: 2-D tiled loads (128-byte swizzle) of the three A
-//               terms and the W k-block into a 3-stage shared-memory ring;
-//   warp 1      allocates 256 TMEM columns and issues tcgen05.mma (one thread);
+//               terms and the W k-block into a shared-memory ring;
+//   warp 1      allocates 512 TMEM columns and issues tcgen05.mma (one thread);
 //               each stage is released by tcgen05.commit to its "empty" barrier;
-//   warps 2..5  tcgen05.ld of their 32 TMEM lanes (one output row per thread),
-//               group sums in registers, then the fused epilogue on column pairs.
+//   warps 2..9  tcgen05.ld of one TMEM lane quadrant and half of the tile's
+//               columns each (one output row per thread), group sums in
+//               registers, then the fused epilogue on column pairs.  The
+//               epilogue of one tile overlaps the MMAs of the next.
 // Every mbarrier wait is bounded; a wait that gives up records its site in
 // *err and the CTA still drains its copies, frees TMEM and exits.
 #pragma once
@@ -33,23 +36,33 @@
 
 namespace wici {
 
-constexpr int TC_BM = 128, TC_BN = 128, TC_BK = 64, TC_STAGES = 3, TC_THREADS = 192;
+constexpr int TC_BM = 128, TC_BK = 64, TC_THREADS = 320, TC_EPI_WARPS = 8;
 constexpr int TC_GROUP = 2;                                             // k-blocks per TMEM accumulation
 constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;                      // 16 KB per term
-constexpr uint32_t TC_B_BYTES = TC_BN * TC_BK * 2;                      // 16 KB
-constexpr uint32_t TC_STAGE_BYTES = kTerms * TC_A_BYTES + TC_B_BYTES;   // 64 KB
-constexpr size_t TC_SMEM = (size_t)TC_STAGES * TC_STAGE_BYTES + 1024;
-constexpr uint32_t TC_TMEM_COLS = 2 * TC_BN;                            // two accumulator buffers
+constexpr uint32_t TC_TMEM_COLS = 512;                                  // two accumulator buffers
+constexpr size_t TC_SMEM_BUDGET = 216 * 1024;                           // ring bytes
+
+// geometry of a 128 x BN output tile
+template <int BN>
+struct TcTile {
+    static_assert(BN % 64 == 0 && BN <= 256, "BN: a multiple of 64 up to 256");
+    static constexpr uint32_t B_BYTES = BN * TC_BK * 2;
+    static constexpr uint32_t STAGE_BYTES = kTerms * TC_A_BYTES + B_BYTES;
+    static constexpr int STAGES = (int)(TC_SMEM_BUDGET / STAGE_BYTES);
+    static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024;
+    static constexpr int EPI_COLS = BN / 2;                               // columns per epilogue warp
+    static_assert(STAGES >= 3, "at least three ring stages");
+};
 
 enum : int { SITE_TC_EMPTY = 21, SITE_TC_FULL = 22, SITE_TC_ACCUM = 23, SITE_TC_DRAIN = 24, SITE_TC_FREE = 25 };
 
 // instruction descriptor of tcgen05.mma.kind::f16: D fp32, A and B bf16, both
-// K-major, M = 128, N = TC_BN
-__host__ __device__ constexpr uint32_t tc_idesc() {
+// K-major, M = 128, N = n
+__host__ __device__ constexpr uint32_t tc_idesc(int n) {
     return (1u << 4)                      // D format: f32
            | (1u << 7)                    // A format: bf16
            | (1u << 10)                   // B format: bf16
-           | ((uint32_t)(TC_BN >> 3) << 17)
+           | ((uint32_t)(n >> 3) << 17)
            | ((uint32_t)(TC_BM >> 4) << 24);
 }
 
@@ -107,31 +120,33 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, float *v) {
 }
 
 // Epi::pair(t, c, v0, v1): output row t, columns (c, c + 1)
-template <class Epi>
+template <int BN, class Epi>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_a1,
                    const __grid_constant__ CUtensorMap map_a2, const __grid_constant__ CUtensorMap map_w, int T,
                    int N, int K, int *err, const Epi epi) {
+    using G = TcTile<BN>;
+    constexpr int S = G::STAGES;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full_bar[TC_STAGES], empty_bar[TC_STAGES], acc_full[2], acc_free[2];
+    __shared__ __align__(8) uint64_t full_bar[S], empty_bar[S], acc_full[2], acc_free[2];
     __shared__ uint32_t s_tmem;
     __shared__ int s_issued;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // M tiles vary fastest: the CTAs that run together share one weight tile through L2
-    const int m0 = blockIdx.x * TC_BM, n0 = blockIdx.y * TC_BN;
+    const int ntm = (T + TC_BM - 1) / TC_BM, ntn = (N + BN - 1) / BN;
+    const int ntiles = ntm * ntn;
     const int nk = (K + TC_BK - 1) / TC_BK;
     const int ngroups = (nk + TC_GROUP - 1) / TC_GROUP;
     const uint32_t base = (smem_u32(smem_raw) + 1023u) & ~1023u;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < TC_STAGES; ++s) {
+        for (int s = 0; s < S; ++s) {
             mbar_init(smem_u32(&full_bar[s]), 1);
             mbar_init(smem_u32(&empty_bar[s]), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&acc_full[b]), 1);
-            mbar_init(smem_u32(&acc_free[b]), 4);
+            mbar_init(smem_u32(&acc_free[b]), TC_EPI_WARPS);
         }
         fence_barrier_init();
         s_issued = 0;
@@ -149,82 +164,94 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
     if (warp == 0) {
         if (lane == 0) {  // ------------------------------------------- TMA producer
-            int issued = 0;
-            for (int kb = 0; kb < nk; ++kb) {
-                const int s = kb % TC_STAGES;
-                if (kb >= TC_STAGES &&
-                    !mbar_wait(smem_u32(&empty_bar[s]), ((kb / TC_STAGES) + 1) & 1, err, SITE_TC_EMPTY))
-                    break;
-                const uint32_t st = base + (uint32_t)s * TC_STAGE_BYTES;
-                const uint32_t fb = smem_u32(&full_bar[s]);
-                mbar_arrive_expect_tx(fb, TC_STAGE_BYTES);
-                tma_load_2d(st, &map_a0, kb * TC_BK, m0, fb);
-                tma_load_2d(st + TC_A_BYTES, &map_a1, kb * TC_BK, m0, fb);
-                tma_load_2d(st + 2 * TC_A_BYTES, &map_a2, kb * TC_BK, m0, fb);
-                tma_load_2d(st + kTerms * TC_A_BYTES, &map_w, kb * TC_BK, n0, fb);
-                issued = kb + 1;
+            int it = 0;   // k-blocks issued over all tiles
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+                const int m0 = (tile % ntm) * TC_BM, n0 = (tile / ntm) * BN;
+                for (int kb = 0; kb < nk; ++kb, ++it) {
+                    const int s = it % S;
+                    if (it >= S && !(ok = mbar_wait(smem_u32(&empty_bar[s]), ((it / S) + 1) & 1, err, SITE_TC_EMPTY)))
+                        break;
+                    const uint32_t st = base + (uint32_t)s * G::STAGE_BYTES;
+                    const uint32_t fb = smem_u32(&full_bar[s]);
+                    mbar_arrive_expect_tx(fb, G::STAGE_BYTES);
+                    tma_load_2d(st, &map_a0, kb * TC_BK, m0, fb);
+                    tma_load_2d(st + TC_A_BYTES, &map_a1, kb * TC_BK, m0, fb);
+                    tma_load_2d(st + 2 * TC_A_BYTES, &map_a2, kb * TC_BK, m0, fb);
+                    tma_load_2d(st + kTerms * TC_A_BYTES, &map_w, kb * TC_BK, n0, fb);
+                    s_issued = it + 1;
+                }
             }
-            s_issued = issued;
         }
     } else if (warp == 1) {
         if (lane == 0) {  // ------------------------------------------- MMA issuer
-            constexpr uint32_t idesc = tc_idesc();
+            constexpr uint32_t idesc = tc_idesc(BN);
             bool ok = true;
-            for (int gi = 0; gi < ngroups && ok; ++gi) {
-                const int b = gi & 1;
-                // the epilogue must have read this buffer's previous group
-                if (gi >= 2 && !(ok = mbar_wait(smem_u32(&acc_free[b]), ((gi / 2) + 1) & 1, err, SITE_TC_FREE)))
-                    break;
-                tc_fence_after();
-                const uint32_t acc = tmem + (uint32_t)(b * TC_BN);
-                const int kb1 = min(nk, (gi + 1) * TC_GROUP);
-                for (int kb = gi * TC_GROUP; kb < kb1; ++kb) {
-                    const int s = kb % TC_STAGES;
-                    ok = mbar_wait(smem_u32(&full_bar[s]), (kb / TC_STAGES) & 1, err, SITE_TC_FULL);
-                    if (!ok) break;
+            int it = 0, gg = 0;   // k-blocks and groups consumed over all tiles
+            for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+                for (int gi = 0; gi < ngroups && ok; ++gi, ++gg) {
+                    const int b = gg & 1;
+                    // the epilogue must have read this buffer's previous group
+                    if (gg >= 2 && !(ok = mbar_wait(smem_u32(&acc_free[b]), ((gg / 2) + 1) & 1, err, SITE_TC_FREE)))
+                        break;
                     tc_fence_after();
-                    const uint32_t st = base + (uint32_t)s * TC_STAGE_BYTES;
+                    const uint32_t acc = tmem + (uint32_t)(b * BN);
+                    const int kb1 = min(nk, (gi + 1) * TC_GROUP);
+                    for (int kb = gi * TC_GROUP; kb < kb1; ++kb, ++it) {
+                        const int s = it % S;
+                        ok = mbar_wait(smem_u32(&full_bar[s]), (it / S) & 1, err, SITE_TC_FULL);
+                        if (!ok) break;
+                        tc_fence_after();
+                        const uint32_t st = base + (uint32_t)s * G::STAGE_BYTES;
+                        // descriptors of k-step 0; each k-step of 16 elements is 32 bytes further
+                        const uint64_t bd0 = tc_desc_sw128(st + kTerms * TC_A_BYTES);
+                        const uint64_t ad0 = tc_desc_sw128(st);
 #pragma unroll
-                    for (int k = 0; k < TC_BK / 16; ++k) {
-                        const uint64_t bd = tc_desc_sw128(st + kTerms * TC_A_BYTES + 32 * k);
+                        for (int k = 0; k < TC_BK / 16; ++k)
 #pragma unroll
-                        for (int t = 0; t < kTerms; ++t)
-                            tc_mma(acc, tc_desc_sw128(st + t * TC_A_BYTES + 32 * k), bd, idesc,
-                                   (kb != gi * TC_GROUP || k != 0 || t != 0));
+                            for (int t = 0; t < kTerms; ++t)
+                                tc_mma(acc, ad0 + (uint64_t)((t * TC_A_BYTES + 32 * k) >> 4), bd0 + (uint64_t)(2 * k),
+                                       idesc, (kb != gi * TC_GROUP || k != 0 || t != 0));
+                        tc_commit(smem_u32(&empty_bar[s]));
                     }
-                    tc_commit(smem_u32(&empty_bar[s]));
+                    tc_commit(smem_u32(&acc_full[b]));  // fires when this group's MMAs have completed
                 }
-                tc_commit(smem_u32(&acc_full[b]));  // fires when this group's MMAs have completed
             }
         }
     } else {  // ------------------------------------------------------- epilogue
-        const int q = warp & 3;                 // TMEM lane quadrant of this warp
-        const int t = m0 + q * 32 + lane;
+        const int q = warp & 3;                          // TMEM lane quadrant of this warp
+        const int half = (warp - 2) >> 2;                // which half of the tile's columns
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-        float sum[TC_BN];
-#pragma unroll
-        for (int c = 0; c < TC_BN; ++c) sum[c] = 0.f;
         bool ok = true;
-        for (int gi = 0; gi < ngroups && ok; ++gi) {
-            const int b = gi & 1;
-            ok = mbar_wait(smem_u32(&acc_full[b]), (gi / 2) & 1, err, SITE_TC_ACCUM);
-            tc_fence_after();
+        int gg = 0;
+        for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+            const int m0 = (tile % ntm) * TC_BM, n0 = (tile / ntm) * BN;
+            const int t = m0 + q * 32 + lane;
+            float sum[G::EPI_COLS];
 #pragma unroll
-            for (int c0 = 0; c0 < TC_BN; c0 += 32) {
-                float v[32];
-                tc_ld32(tmem + lane_base + (uint32_t)(b * TC_BN + c0), v);
+            for (int c = 0; c < G::EPI_COLS; ++c) sum[c] = 0.f;
+            for (int gi = 0; gi < ngroups; ++gi, ++gg) {
+                const int b = gg & 1;
+                ok = mbar_wait(smem_u32(&acc_full[b]), (gg / 2) & 1, err, SITE_TC_ACCUM);
+                if (!ok) break;
+                tc_fence_after();
 #pragma unroll
-                for (int i = 0; i < 32; ++i) sum[c0 + i] += v[i];
+                for (int c0 = 0; c0 < G::EPI_COLS; c0 += 32) {
+                    float v[32];
+                    tc_ld32(tmem + lane_base + (uint32_t)(b * BN + half * G::EPI_COLS + c0), v);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) sum[c0 + i] += v[i];
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&acc_free[b]));
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&acc_free[b]));
-        }
-        if (ok && t < T) {
+            if (ok && t < T) {
 #pragma unroll
-            for (int j = 0; j < TC_BN; j += 2) {
-                const int c = n0 + j;
-                if (c < N) epi.pair(t, c, sum[j], sum[j + 1]);
+                for (int j = 0; j < G::EPI_COLS; j += 2) {
+                    const int c = n0 + half * G::EPI_COLS + j;
+                    if (c < N) epi.pair(t, c, sum[j], sum[j + 1]);
+                }
             }
         }
     }
@@ -234,8 +261,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         // nothing may still land in shared memory after exit (all stages were
         // consumed on the normal path; this only matters after a wait gave up)
         const int issued = s_issued;
-        for (int kb = issued - TC_STAGES < 0 ? 0 : issued - TC_STAGES; kb < issued; ++kb)
-            mbar_wait(smem_u32(&full_bar[kb % TC_STAGES]), (kb / TC_STAGES) & 1, err, SITE_TC_DRAIN);
+        for (int kb = issued - S < 0 ? 0 : issued - S; kb < issued; ++kb)
+            mbar_wait(smem_u32(&full_bar[kb % S]), (kb / S) & 1, err, SITE_TC_DRAIN);
     }
     if (warp == 1) {
         tc_fence_after();

@@ -740,6 +740,7 @@ __global__ void __launch_bounds__(32 * (kFdMaxQueryWarps + 1)) flash_decode_kern
 constexpr int kMegaSlots = 6;
 constexpr uint32_t kMegaSlotBytes = 32768;
 constexpr size_t kMegaSmem = kGemvRedBytes + (size_t)kMegaSlots * kMegaSlotBytes;
+constexpr size_t kMegaPrefetchBytes = 196608;   // gate/up bytes per CTA moved into L2 during attention
 
 enum : int { SITE_MEGA_EMPTY = 51, SITE_MEGA_FULL = 52, SITE_MEGA_DRAIN = 53, SITE_MEGA_GRID = 54 };
 
@@ -800,6 +801,19 @@ __device__ bool mp_rows(MegaRing &R, const uint16_t *W, int K, int n_units, int 
     return true;
 }
 
+// move rows [skip, skip + bytes) of this CTA's share of a GEMV phase into L2
+__device__ void mp_prefetch(const uint16_t *W, int K, int n_units, int rpu, size_t skip, size_t bytes) {
+    const int u0 = mega_u0(n_units);
+    const int u1 = (int)(((long long)(blockIdx.x + 1) * n_units) / gridDim.x);
+    const size_t row = (size_t)K * 2;
+    const size_t own = (size_t)(u1 - u0) * rpu * row;
+    skip -= skip % row;
+    const size_t end = own < skip + bytes ? own : skip + bytes;
+    const uint8_t *src = reinterpret_cast<const uint8_t *>(W + (size_t)u0 * rpu * K);
+    for (size_t off = skip; off < end; off += 32768)
+        bulk_prefetch_l2(src + off, (uint32_t)(end - off < 32768 ? end - off : 32768));
+}
+
 // the pages of this CTA's attention split (its K and V blocks), one page per slot
 struct MegaSplit {
     int g, r, p0, n, npages, splits;
@@ -850,8 +864,9 @@ __device__ bool mega_grid_sync(int *ctrl, int k, int *s_flag) {
     if (threadIdx.x == 0) {
         int *ctr = ctrl + CTRL_GRID_BAR;
         const int target = k * (int)gridDim.x;
-        __threadfence();
-        atomicAdd(ctr, 1);
+        // release: every consumer store of this CTA (ordered before this thread by
+        // the barrier above) is visible to a CTA whose acquire load sees the count
+        asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(ctr) : "memory");
         bool ok = false;
         const uint64_t t0 = globaltimer_ns();
         for (uint32_t it = 0; it < 0x7FFFFFFFu; ++it) {
@@ -868,7 +883,6 @@ __device__ bool mega_grid_sync(int *ctrl, int k, int *s_flag) {
             }
             __nanosleep(20);
         }
-        __threadfence();
         *s_flag = ok ? 1 : 0;
     }
     consumer_sync();
@@ -1283,8 +1297,12 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
         eq.qdim = a.qdim; eq.kvdim = a.kvdim; eq.d = a.d; eq.nkv = a.nkv; eq.page_elems = a.page_elems;
         ok = mc_gemv<SH>(R, red, a.H, a.nqkv / 2, 2, a.x, a.W + a.l0.attn_norm + lo,
                          l == 0 ? a.W + a.w_embed : nullptr, a.x, a.eps, a.ctrl, eq, s_part) &&
-             mega_grid_sync(a.ctrl, ++k, &s_flag) &&
-             mc_attn<D>(R, a, kvl, sp, len, s_state, &s_last) &&
+             mega_grid_sync(a.ctrl, ++k, &s_flag);
+        if (!ok) break;
+        // the attention phase leaves the HBM nearly idle: move the first gate/up rows
+        // of this CTA into L2 meanwhile (its O rows are already filling the ring)
+        if (tid == 0) mp_prefetch(a.W + a.l0.wgu + lo, a.H, a.F, 2, 0, kMegaPrefetchBytes);
+        ok = mc_attn<D>(R, a, kvl, sp, len, s_state, &s_last) &&
              mega_grid_sync(a.ctrl, ++k, &s_flag);
         if (!ok) break;
         EpiResidual er{a.x};

@@ -15,6 +15,9 @@
 
 namespace wici {
 
+// output-tile width of the prefill GEMMs: 128 x 192 tiles, three 72 KB ring stages
+constexpr int kPrefillBN = 192;
+
 // store a as its three bf16 terms
 __device__ __forceinline__ void split_store(uint16_t *const *t, size_t i, float a) {
     uint16_t t0, t1, t2;
@@ -201,20 +204,21 @@ const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
     m->wd.resize(p.L);
     for (int l = 0; l < p.L; ++l) {
         const LayerOffsets &lo = p.layer[l];
-        ok = encode_2d(&m->wqkv[l], b.W + lo.wqkv, p.nqkv, p.H, TC_BN) &&
-             encode_2d(&m->wo[l], b.W + lo.wo, p.H, p.qdim, TC_BN) &&
-             encode_2d(&m->wgu[l], b.W + lo.wgu, 2 * p.F, p.H, TC_BN) &&
-             encode_2d(&m->wd[l], b.W + lo.wd, p.H, p.F, TC_BN);
+        ok = encode_2d(&m->wqkv[l], b.W + lo.wqkv, p.nqkv, p.H, kPrefillBN) &&
+             encode_2d(&m->wo[l], b.W + lo.wo, p.H, p.qdim, kPrefillBN) &&
+             encode_2d(&m->wgu[l], b.W + lo.wgu, 2 * p.F, p.H, kPrefillBN) &&
+             encode_2d(&m->wd[l], b.W + lo.wd, p.H, p.F, kPrefillBN);
         if (!ok) return "cuTensorMapEncodeTiled failed for a weight matrix";
     }
     static bool attrs = false;
     if (!attrs) {
-        if (cudaFuncSetAttribute(gemm_tc_kernel<PEpiQKV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)TC_SMEM) != cudaSuccess ||
-            cudaFuncSetAttribute(gemm_tc_kernel<PEpiResidual>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)TC_SMEM) != cudaSuccess ||
-            cudaFuncSetAttribute(gemm_tc_kernel<PEpiSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)TC_SMEM) != cudaSuccess ||
+        constexpr int smem = (int)TcTile<kPrefillBN>::SMEM;
+        if (cudaFuncSetAttribute(gemm_tc_kernel<kPrefillBN, PEpiQKV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 smem) != cudaSuccess ||
+            cudaFuncSetAttribute(gemm_tc_kernel<kPrefillBN, PEpiResidual>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+            cudaFuncSetAttribute(gemm_tc_kernel<kPrefillBN, PEpiSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 smem) != cudaSuccess ||
             cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)(AttnSmem<128>::TOTAL + 1024)) != cudaSuccess ||
             cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -251,11 +255,13 @@ cudaError_t launch_attn_tc(const Plan &p, const Bufs &b, const PrefillMaps &mp, 
 }
 
 template <class Epi>
-static cudaError_t gemm(const CUtensorMap *a, const CUtensorMap &w, int T, int N, int K, int *err, const Epi &epi,
-                        cudaStream_t st, LaunchHook *hook, const char *name) {
+static cudaError_t gemm(const Plan &p, const CUtensorMap *a, const CUtensorMap &w, int T, int N, int K, int *err,
+                        const Epi &epi, cudaStream_t st, LaunchHook *hook, const char *name) {
     if (hook) hook->before(name);
-    dim3 grid((T + TC_BM - 1) / TC_BM, (N + TC_BN - 1) / TC_BN);
-    gemm_tc_kernel<Epi><<<grid, TC_THREADS, TC_SMEM, st>>>(a[0], a[1], a[2], w, T, N, K, err, epi);
+    const int tiles = ((T + TC_BM - 1) / TC_BM) * ((N + kPrefillBN - 1) / kPrefillBN);
+    const int grid = tiles < p.num_sms ? tiles : p.num_sms;   // persistent: at most one CTA per SM
+    gemm_tc_kernel<kPrefillBN, Epi><<<grid, TC_THREADS, TcTile<kPrefillBN>::SMEM, st>>>(a[0], a[1], a[2], w, T, N, K,
+                                                                                        err, epi);
     if (hook) hook->after(name);
     return cudaGetLastError();
 }
@@ -274,7 +280,7 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.attn_norm, A, p.H, p.cfg.rms_eps);
         PEpiQKV eq = {{{b.Q[0], b.Q[1], b.Q[2]}}, kvl, b.pages, b.rope, p.cfg.qkv_bias ? b.W + lo.bqkv : nullptr, P, p.qdim,
                       p.kvdim, p.d, p.nkv, p.kv_page_elems};
-        if ((e = gemm(mp.a, mp.wqkv[l], T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
+        if ((e = gemm(p, mp.a, mp.wqkv[l], T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
             return e;
         // A5: causal attention over the cache (earlier chunks + this one), tensor cores
         if (hook) hook->before("prefill_attention");
@@ -282,17 +288,17 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         if (hook) hook->after("prefill_attention");
         if (e != cudaSuccess) return e;
         // A6: O projection + residual
-        if ((e = gemm(mp.o, mp.wo[l], T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
+        if ((e = gemm(p, mp.o, mp.wo[l], T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_o_proj")) != cudaSuccess)
             return e;
         // A7: RMSNorm + gate/up + SwiGLU
         rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.ffn_norm, A, p.H, p.cfg.rms_eps);
         const Terms M = {{b.M[0], b.M[1], b.M[2]}};
-        if ((e = gemm(mp.a, mp.wgu[l], T, 2 * p.F, p.H, err, PEpiSwiGLU{M, p.F}, st, hook,
+        if ((e = gemm(p, mp.a, mp.wgu[l], T, 2 * p.F, p.H, err, PEpiSwiGLU{M, p.F}, st, hook,
                       "prefill_gate_up")) != cudaSuccess)
             return e;
         // A8: down projection + residual
-        if ((e = gemm(mp.m, mp.wd[l], T, p.H, p.F, err, PEpiResidual{b.X, p.H}, st, hook,
+        if ((e = gemm(p, mp.m, mp.wd[l], T, p.H, p.F, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_down")) != cudaSuccess)
             return e;
     }
