@@ -119,7 +119,8 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, float *v) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Epi::pair(t, c, v0, v1): output row t, columns (c, c + 1)
+// Epi::pair(t, c, v0, v1): output row t, columns (c, c + 1); Epi::row (when
+// Epi::kRow): the thread's whole span of columns at once, with vector stores
 template <int BN, class Epi>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_a1,
@@ -247,10 +248,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                 if (lane == 0) mbar_arrive(smem_u32(&acc_free[b]));
             }
             if (ok && t < T) {
+                const int c0 = n0 + half * G::EPI_COLS;
+                if constexpr (Epi::kRow) {
+                    epi.row(t, c0, sum, N - c0);
+                } else {
 #pragma unroll
-                for (int j = 0; j < G::EPI_COLS; j += 2) {
-                    const int c = n0 + half * G::EPI_COLS + j;
-                    if (c < N) epi.pair(t, c, sum[j], sum[j + 1]);
+                    for (int j = 0; j < G::EPI_COLS; j += 2)
+                        if (c0 + j < N) epi.pair(t, c0 + j, sum[j], sum[j + 1]);
                 }
             }
         }

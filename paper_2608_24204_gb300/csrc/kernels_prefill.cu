@@ -58,6 +58,7 @@ __global__ void rmsnorm_rows_kernel(const float *X, const uint16_t *g, const Ter
 // --------------------------------------------------------------- epilogues ----
 // pair(t, c, a, b): GEMM output row t, columns (c, c + 1)
 struct PEpiQKV {  // packed QKV columns -> Q (three bf16 terms) and K/V pages (bf16)
+    static constexpr bool kRow = true;
     Terms Q;
     uint16_t *kv;
     const int *pages;
@@ -94,11 +95,87 @@ struct PEpiQKV {  // packed QKV columns -> Q (three bf16 terms) and K/V pages (b
             vr[e + 1] = f32_to_bf16(b);
         }
     }
+    // 16 columns at a time: one head and one of q / k / v (head_dim, qdim and
+    // kvdim are multiples of 64), 16-byte stores
+    template <int NC>
+    __device__ __forceinline__ void row(int t, int c0, const float (&v)[NC], int n) const {
+        const int pos = P + t;
+        uint16_t *page = kv + (size_t)pages[pos / kPage] * page_elems;
+        const int slot = pos % kPage, half = d >> 1;
+#pragma unroll
+        for (int g = 0; g < NC; g += 16) {
+            const int c = c0 + g;
+            if (g + 16 > n) {
+#pragma unroll
+                for (int k = 0; k < 16; k += 2)
+                    if (g + k + 1 < n) pair(t, c + k, v[g + k], v[g + k + 1]);
+                continue;
+            }
+            float x[16];
+#pragma unroll
+            for (int k = 0; k < 16; ++k) x[k] = v[g + k] + (bias ? bf16_to_f32(bias[c + k]) : 0.f);
+            if (c < qdim + kvdim) {
+                const int hd = c / d, i0 = (c % d) >> 1;
+                float ra[8], rb[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const float2 cs = rope[(size_t)pos * half + i0 + k];
+                    ra[k] = x[2 * k] * cs.x - x[2 * k + 1] * cs.y;
+                    rb[k] = x[2 * k + 1] * cs.x + x[2 * k] * cs.y;
+                }
+                if (c < qdim) {
+                    const size_t qo = (size_t)t * qdim + hd * d + i0;
+                    uint32_t wa[kTerms][4], wb[kTerms][4];
+#pragma unroll
+                    for (int k = 0; k < 8; k += 2) {
+                        uint16_t a0[kTerms], a1[kTerms], b0[kTerms], b1[kTerms];
+                        split_bf16x3(ra[k], a0[0], a0[1], a0[2]);
+                        split_bf16x3(ra[k + 1], a1[0], a1[1], a1[2]);
+                        split_bf16x3(rb[k], b0[0], b0[1], b0[2]);
+                        split_bf16x3(rb[k + 1], b1[0], b1[1], b1[2]);
+#pragma unroll
+                        for (int q = 0; q < kTerms; ++q) {
+                            wa[q][k >> 1] = (uint32_t)a0[q] | ((uint32_t)a1[q] << 16);
+                            wb[q][k >> 1] = (uint32_t)b0[q] | ((uint32_t)b1[q] << 16);
+                        }
+                    }
+#pragma unroll
+                    for (int q = 0; q < kTerms; ++q) {
+                        *reinterpret_cast<uint4 *>(Q.p[q] + qo) = make_uint4(wa[q][0], wa[q][1], wa[q][2], wa[q][3]);
+                        *reinterpret_cast<uint4 *>(Q.p[q] + qo + half) =
+                            make_uint4(wb[q][0], wb[q][1], wb[q][2], wb[q][3]);
+                    }
+                } else {
+                    uint16_t *kr = page + ((size_t)(hd - qdim / d) * kPage + slot) * d + i0;
+                    uint32_t wa[4], wb[4];
+#pragma unroll
+                    for (int k = 0; k < 8; k += 2) {
+                        wa[k >> 1] = (uint32_t)f32_to_bf16(ra[k]) | ((uint32_t)f32_to_bf16(ra[k + 1]) << 16);
+                        wb[k >> 1] = (uint32_t)f32_to_bf16(rb[k]) | ((uint32_t)f32_to_bf16(rb[k + 1]) << 16);
+                    }
+                    *reinterpret_cast<uint4 *>(kr) = make_uint4(wa[0], wa[1], wa[2], wa[3]);
+                    *reinterpret_cast<uint4 *>(kr + half) = make_uint4(wb[0], wb[1], wb[2], wb[3]);
+                }
+            } else {
+                const int j = c - qdim - kvdim, vh = j / d, e0 = j % d;
+                uint16_t *vr = page + (size_t)nkv * kPage * d + ((size_t)vh * kPage + slot) * d + e0;
+                uint32_t w[8];
+#pragma unroll
+                for (int k = 0; k < 16; k += 2)
+                    w[k >> 1] = (uint32_t)f32_to_bf16(x[k]) | ((uint32_t)f32_to_bf16(x[k + 1]) << 16);
+                *reinterpret_cast<uint4 *>(vr) = make_uint4(w[0], w[1], w[2], w[3]);
+                *reinterpret_cast<uint4 *>(vr + 8) = make_uint4(w[4], w[5], w[6], w[7]);
+            }
+        }
+    }
 };
 
+// row(t, c0, v, n): output row t, columns c0 .. c0 + n of one thread's span
+// (NC consecutive columns, c0 a multiple of 32), written with 16-byte stores
 struct PEpiResidual {  // X[t][c] += v
     float *X;
     int ld;
+    static constexpr bool kRow = true;
     __device__ void pair(int t, int c, float a, float b) const {
         float2 *p = reinterpret_cast<float2 *>(X + (size_t)t * ld + c);
         float2 v = *p;
@@ -106,13 +183,58 @@ struct PEpiResidual {  // X[t][c] += v
         v.y += b;
         *p = v;
     }
+    template <int NC>
+    __device__ __forceinline__ void row(int t, int c0, const float (&v)[NC], int n) const {
+        float *x = X + (size_t)t * ld + c0;
+#pragma unroll
+        for (int j = 0; j < NC; j += 4) {
+            if (j + 4 <= n) {
+                float4 *p = reinterpret_cast<float4 *>(x + j);
+                float4 a = *p;
+                a.x += v[j]; a.y += v[j + 1]; a.z += v[j + 2]; a.w += v[j + 3];
+                *p = a;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (j + e < n) x[j + e] += v[j + e];
+            }
+        }
+    }
 };
 
 struct PEpiSwiGLU {  // interleaved (gate, up) columns -> M[t][c/2] = silu(g) * u as three terms
     Terms M;
     int ld;
+    static constexpr bool kRow = true;
     __device__ void pair(int t, int c, float a, float b) const {
         split_store(M.p, (size_t)t * ld + (c >> 1), a / (1.0f + expf(-a)) * b);
+    }
+    template <int NC>
+    __device__ __forceinline__ void row(int t, int c0, const float (&v)[NC], int n) const {
+        const size_t o = (size_t)t * ld + (c0 >> 1);
+#pragma unroll
+        for (int j = 0; j < NC; j += 16) {   // 8 outputs: one 16-byte store per term
+            if (j + 16 <= n) {
+                uint32_t w[kTerms][4];
+#pragma unroll
+                for (int k = 0; k < 8; k += 2) {
+                    const float g0 = v[j + 2 * k], u0 = v[j + 2 * k + 1];
+                    const float g1 = v[j + 2 * k + 2], u1 = v[j + 2 * k + 3];
+                    uint16_t a[kTerms], b[kTerms];
+                    split_bf16x3(g0 / (1.0f + expf(-g0)) * u0, a[0], a[1], a[2]);
+                    split_bf16x3(g1 / (1.0f + expf(-g1)) * u1, b[0], b[1], b[2]);
+#pragma unroll
+                    for (int q = 0; q < kTerms; ++q) w[q][k >> 1] = (uint32_t)a[q] | ((uint32_t)b[q] << 16);
+                }
+#pragma unroll
+                for (int q = 0; q < kTerms; ++q)
+                    *reinterpret_cast<uint4 *>(M.p[q] + o + (j >> 1)) = make_uint4(w[q][0], w[q][1], w[q][2], w[q][3]);
+            } else {
+#pragma unroll
+                for (int k = 0; k < 16; k += 2)
+                    if (j + k + 1 < n) pair(t, c0 + j + k, v[j + k], v[j + k + 1]);
+            }
+        }
     }
 };
 
