@@ -24,6 +24,8 @@ struct Bufs {
     float *logits;    // last logits                                        [V]
     int2 *amax;       // per-CTA argmax partials (value bits, index)        [num_sms]
     float *fd_part;   // flash-decode split states                           [nkv][splits][group][d + 4]
+    uint32_t *mega_bound; // persistent decode: row-share boundaries (2^24 = all) [num_sms + 1]
+    float *mega_time;     // persistent decode: gate/up time per CTA, last step (us) [num_sms]
     float2 *rope;     // (cos, sin) of p * theta^(-2i/d)                     [max_tokens][d/2]
     int *pages;       // logical -> physical KV page                         [max_pages]
     int *tok;         // prefill chunk tokens                                [max_chunk]
@@ -40,7 +42,8 @@ struct PrefillMaps {
     CUtensorMap a[kTerms], o[kTerms], m[kTerms];       // GEMM activations, 128-row boxes
     CUtensorMap q[kTerms];                             // queries: [token][head][d], group x tpt boxes
     CUtensorMap kv;                                    // the whole KV pool: [page][K|V][kv_head][16][d]
-    std::vector<CUtensorMap> wqkv, wo, wgu, wd;        // per layer weights, 256-row boxes
+    std::vector<CUtensorMap> wqkv, wo, wgu, wd;        // per layer weights, boxes of bn_* rows
+    int bn_qkv, bn_o, bn_gu, bn_d;                     // output-tile width of each matrix's GEMM
 };
 
 // Encodes every tensor map of `m`; returns an error message or nullptr.

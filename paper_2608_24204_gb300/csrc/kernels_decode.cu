@@ -740,7 +740,8 @@ __global__ void __launch_bounds__(32 * (kFdMaxQueryWarps + 1)) flash_decode_kern
 constexpr int kMegaSlots = 6;
 constexpr uint32_t kMegaSlotBytes = 32768;
 constexpr size_t kMegaSmem = kGemvRedBytes + (size_t)kMegaSlots * kMegaSlotBytes;
-constexpr size_t kMegaPrefetchBytes = 196608;   // gate/up bytes per CTA moved into L2 during attention
+constexpr size_t kMegaPrefetchBytes = 196608;
+constexpr int kMegaMaxCtas = 256;   // grid size limit (one CTA per SM)   // gate/up bytes per CTA moved into L2 during attention
 
 enum : int { SITE_MEGA_EMPTY = 51, SITE_MEGA_FULL = 52, SITE_MEGA_DRAIN = 53, SITE_MEGA_GRID = 54 };
 
@@ -763,6 +764,8 @@ struct MegaArgs {
     const float2 *rope;
     const int *pages;
     float *part;                // attention split states [nkv][splits][group][d + 4]
+    uint32_t *bound;            // [grid + 1] share boundaries of the GEMV phases (2^24 = all rows)
+    float *cta_time;            // [grid] each CTA's gate/up streaming time in the last step (us)
     int L, H, F, V, nqkv, qdim, kvdim, d, nkv, group, wph, splits;
     int bias;
     float eps, qscale;
@@ -773,17 +776,19 @@ struct MegaRing {
     const uint8_t *ring;             // generic pointer to slot 0
     int n;   // slots issued (producer) or consumed (consumer) so far
     int *abort;                      // shared flag: a consumer wait gave up
+    uint32_t b0, b1;                 // this CTA's share of every GEMV phase: [b0, b1) / 2^24
 };
 
-__device__ __forceinline__ int mega_u0(int n_units) {
-    return (int)(((long long)blockIdx.x * n_units) / gridDim.x);
+// units [u0, u1) of an n-unit phase for the share [b0, b1) (fixed point, 2^24 = all)
+__device__ __forceinline__ int mega_unit(uint32_t b, int n_units) {
+    return (int)(((unsigned long long)b * (unsigned long long)n_units) >> 24);
 }
 
 // ----------------------------------------------------------- producer side --
 __device__ bool mp_rows(MegaRing &R, const uint16_t *W, int K, int n_units, int rpu, int RPS, int *err,
                         uint64_t pol) {
-    const int u0 = mega_u0(n_units);
-    const int u1 = (int)(((long long)(blockIdx.x + 1) * n_units) / gridDim.x);
+    const int u0 = mega_unit(R.b0, n_units);
+    const int u1 = mega_unit(R.b1, n_units);
     const int total_rows = (u1 - u0) * rpu;
     const int nst = (total_rows + RPS - 1) / RPS;
     const uint16_t *src = W + (size_t)u0 * rpu * K;
@@ -802,9 +807,10 @@ __device__ bool mp_rows(MegaRing &R, const uint16_t *W, int K, int n_units, int 
 }
 
 // move rows [skip, skip + bytes) of this CTA's share of a GEMV phase into L2
-__device__ void mp_prefetch(const uint16_t *W, int K, int n_units, int rpu, size_t skip, size_t bytes) {
-    const int u0 = mega_u0(n_units);
-    const int u1 = (int)(((long long)(blockIdx.x + 1) * n_units) / gridDim.x);
+__device__ void mp_prefetch(const MegaRing &R, const uint16_t *W, int K, int n_units, int rpu, size_t skip,
+                            size_t bytes) {
+    const int u0 = mega_unit(R.b0, n_units);
+    const int u1 = mega_unit(R.b1, n_units);
     const size_t row = (size_t)K * 2;
     const size_t own = (size_t)(u1 - u0) * rpu * row;
     skip -= skip % row;
@@ -898,8 +904,8 @@ __device__ bool mc_gemv(MegaRing &R, float *red, int K, int n_units, int rpu, co
     constexpr int NCH = SH::NCH, RPS = SH::RPS;
     constexpr bool FULL = SH::FULL;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int u0 = mega_u0(n_units);
-    const int u1 = (int)(((long long)(blockIdx.x + 1) * n_units) / gridDim.x);
+    const int u0 = mega_unit(R.b0, n_units);
+    const int u1 = mega_unit(R.b1, n_units);
     const int total_rows = (u1 - u0) * rpu;
     const int nst = (total_rows + RPS - 1) / RPS;
     int *err = ctrl + CTRL_ERR;
@@ -1229,6 +1235,43 @@ __device__ bool mc_attn(MegaRing &R, const MegaArgs &a, const uint16_t *kvl, con
     return true;
 }
 
+// The SMs do not draw equal HBM bandwidth, and which SMs are slow stays the same
+// from step to step, so the GEMV rows are split in proportion to each CTA's
+// measured speed instead of evenly.  Run by the consumers of the last CTA of a
+// step: the new share of CTA b blends its old share with old share / time of
+// its gate/up phases (normalised), half and half, with a floor of a quarter of
+// an even share.  Which CTA streams which rows changes no result.
+__device__ void mega_rebalance(const MegaArgs &a, float *rate) {
+    const int G = gridDim.x, tid = threadIdx.x;
+    for (int b = tid; b < G; b += kGemvConsumers) {
+        const float share = (float)(__ldcg(a.bound + b + 1) - __ldcg(a.bound + b)) * (1.0f / 16777216.0f);
+        const float t = __ldcg(a.cta_time + b);
+        rate[b] = t > 0.f ? share / t : 0.f;
+        rate[kMegaMaxCtas + b] = share;
+    }
+    consumer_sync();
+    if (tid == 0) {
+        float tot = 0.f;
+        for (int b = 0; b < G; ++b) tot += rate[b];
+        if (tot > 0.f) {
+            const float floor_share = 0.25f / (float)G;
+            float sum = 0.f;
+            for (int b = 0; b < G; ++b) {
+                const float ns = fmaxf(0.5f * rate[kMegaMaxCtas + b] + 0.5f * rate[b] / tot, floor_share);
+                rate[b] = ns;
+                sum += ns;
+            }
+            float acc = 0.f;
+            a.bound[0] = 0;
+            for (int b = 1; b < G; ++b) {
+                acc += rate[b - 1] / sum;
+                a.bound[b] = (uint32_t)fminf(acc * 16777216.0f, 16777216.0f);
+            }
+            a.bound[G] = 1u << 24;
+        }
+    }
+}
+
 template <int D, class SH, class SF>
 __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const MegaArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -1239,6 +1282,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
     __shared__ float s_bv[kGemvWarps];
     __shared__ int s_bi[kGemvWarps];
     __shared__ int s_flag, s_last, s_abort;
+    __shared__ float s_part_rate[2 * kMegaMaxCtas];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     int *err = a.ctrl + CTRL_ERR;
 
@@ -1249,6 +1293,9 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
     R.ring = smem + kGemvRedBytes;
     R.n = 0;
     R.abort = &s_abort;
+    // the table changes only at the very end of a step, after every CTA read it here
+    R.b0 = a.bound[blockIdx.x];
+    R.b1 = a.bound[blockIdx.x + 1];
     if (tid == 0) {
         s_abort = 0;
         for (int s = 0; s < kMegaSlots; ++s) {
@@ -1286,6 +1333,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
     // ---------------------------------------------------------------- consumers
     int k = 0;   // grid barriers passed
     bool ok = true;
+    uint64_t gu_ns = 0;   // this CTA's time in the gate/up phases (thread 0's clock)
     for (int l = 0; l < a.L && ok; ++l) {
         const size_t lo = (size_t)l * a.lstride;
         uint16_t *kvl = a.KV + (size_t)l * a.kv_layer_elems;
@@ -1301,7 +1349,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
         if (!ok) break;
         // the attention phase leaves the HBM nearly idle: move the first gate/up rows
         // of this CTA into L2 meanwhile (its O rows are already filling the ring)
-        if (tid == 0) mp_prefetch(a.W + a.l0.wgu + lo, a.H, a.F, 2, 0, kMegaPrefetchBytes);
+        if (tid == 0) mp_prefetch(R, a.W + a.l0.wgu + lo, a.H, a.F, 2, 0, kMegaPrefetchBytes);
         ok = mc_attn<D>(R, a, kvl, sp, len, s_state, &s_last) &&
              mega_grid_sync(a.ctrl, ++k, &s_flag);
         if (!ok) break;
@@ -1310,12 +1358,15 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
              mega_grid_sync(a.ctrl, ++k, &s_flag);
         if (!ok) break;
         EpiSwiGLU es{a.m};
+        const uint64_t t_gu = globaltimer_ns();
         ok = mc_gemv<SH>(R, red, a.H, a.F, 2, a.x, a.W + a.l0.ffn_norm + lo, nullptr, nullptr, a.eps, a.ctrl, es,
-                         s_part) &&
-             mega_grid_sync(a.ctrl, ++k, &s_flag);
+                         s_part);
+        gu_ns += globaltimer_ns() - t_gu;
+        ok = ok && mega_grid_sync(a.ctrl, ++k, &s_flag);
         if (!ok) break;
         ok = mc_gemv<SF>(R, red, a.F, a.H, 1, a.m, nullptr, nullptr, nullptr, a.eps, a.ctrl, er, s_part);
     }
+    if (tid == 0) a.cta_time[blockIdx.x] = (float)gu_ns * 1e-3f;
     if (ok) ok = mega_grid_sync(a.ctrl, ++k, &s_flag);
     if (!ok) return;
     EpiArgmax ea;
@@ -1356,7 +1407,10 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
             a.hist[np] = fi;
             a.ctrl[CTRL_LM_TICKET] = 0;
         }
+        s_last = (t == (int)gridDim.x - 1);
     }
+    consumer_sync();
+    if (s_last) mega_rebalance(a, s_part_rate);
 }
 
 // ------------------------------------------------------------ probe kernel ----
@@ -1599,7 +1653,7 @@ static bool shape_is(int K) {
 }
 
 static MegaLaunch mega_launcher(const Plan &p) {
-    if (p.qdim != p.H || p.nkv > 64) return nullptr;
+    if (p.qdim != p.H || p.nkv > 64 || p.num_sms > kMegaMaxCtas) return nullptr;
     // every layer's tensors must sit at one fixed stride
     if (p.L > 1) {
         const size_t st = p.layer[1].wqkv - p.layer[0].wqkv;
@@ -1639,6 +1693,8 @@ static cudaError_t enqueue_mega(const Plan &p, const Bufs &b, cudaStream_t st, M
     a.rope = b.rope;
     a.pages = b.pages;
     a.part = b.fd_part;
+    a.bound = b.mega_bound;
+    a.cta_time = b.mega_time;
     a.L = p.L; a.H = p.H; a.F = p.F; a.V = p.V;
     a.nqkv = p.nqkv; a.qdim = p.qdim; a.kvdim = p.kvdim; a.d = p.d; a.nkv = p.nkv; a.group = p.group;
     a.wph = fd_wph(p.group);

@@ -15,8 +15,16 @@
 
 namespace wici {
 
-// output-tile width of the prefill GEMMs: 128 x 192 tiles, three 72 KB ring stages
-constexpr int kPrefillBN = 192;
+// output-tile widths of the prefill GEMMs: 128 x 192 tiles (three 72 KB ring
+// stages) or 128 x 128 tiles (three 64 KB stages), chosen per weight matrix
+// for the fewest whole waves of tiles at the largest chunk
+static int pick_bn(int T, int N, int sms) {
+    const int tm = (T + TC_BM - 1) / TC_BM;
+    const int w192 = (tm * ((N + 191) / 192) + sms - 1) / sms;
+    const int w128 = (tm * ((N + 127) / 128) + sms - 1) / sms;
+    // a narrower tile reads its A operand more often per FLOP: charge it 10%
+    return (double)w128 * 128 * 1.1 < (double)w192 * 192 ? 128 : 192;
+}
 
 // store a as its three bf16 terms
 __device__ __forceinline__ void split_store(uint16_t *const *t, size_t i, float a) {
@@ -320,27 +328,34 @@ const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
     if (!ok) return "cuTensorMapEncodeTiled failed for an activation operand";
     ok = encode_kv(&m->kv, b.KV, p);
     if (!ok) return "cuTensorMapEncodeTiled failed for the attention operands";
+    m->bn_qkv = pick_bn(T, p.nqkv, p.num_sms);
+    m->bn_o = pick_bn(T, p.H, p.num_sms);
+    m->bn_gu = pick_bn(T, 2 * p.F, p.num_sms);
+    m->bn_d = pick_bn(T, p.H, p.num_sms);
     m->wqkv.resize(p.L);
     m->wo.resize(p.L);
     m->wgu.resize(p.L);
     m->wd.resize(p.L);
     for (int l = 0; l < p.L; ++l) {
         const LayerOffsets &lo = p.layer[l];
-        ok = encode_2d(&m->wqkv[l], b.W + lo.wqkv, p.nqkv, p.H, kPrefillBN) &&
-             encode_2d(&m->wo[l], b.W + lo.wo, p.H, p.qdim, kPrefillBN) &&
-             encode_2d(&m->wgu[l], b.W + lo.wgu, 2 * p.F, p.H, kPrefillBN) &&
-             encode_2d(&m->wd[l], b.W + lo.wd, p.H, p.F, kPrefillBN);
+        ok = encode_2d(&m->wqkv[l], b.W + lo.wqkv, p.nqkv, p.H, m->bn_qkv) &&
+             encode_2d(&m->wo[l], b.W + lo.wo, p.H, p.qdim, m->bn_o) &&
+             encode_2d(&m->wgu[l], b.W + lo.wgu, 2 * p.F, p.H, m->bn_gu) &&
+             encode_2d(&m->wd[l], b.W + lo.wd, p.H, p.F, m->bn_d);
         if (!ok) return "cuTensorMapEncodeTiled failed for a weight matrix";
     }
     static bool attrs = false;
     if (!attrs) {
-        constexpr int smem = (int)TcTile<kPrefillBN>::SMEM;
-        if (cudaFuncSetAttribute(gemm_tc_kernel<kPrefillBN, PEpiQKV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 smem) != cudaSuccess ||
-            cudaFuncSetAttribute(gemm_tc_kernel<kPrefillBN, PEpiResidual>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
-            cudaFuncSetAttribute(gemm_tc_kernel<kPrefillBN, PEpiSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 smem) != cudaSuccess ||
+        constexpr int s192 = (int)TcTile<192>::SMEM, s128 = (int)TcTile<128>::SMEM;
+        const auto attr = [](const void *f, int bytes) {
+            return cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) == cudaSuccess;
+        };
+        if (!attr((const void *)gemm_tc_kernel<192, PEpiQKV>, s192) ||
+            !attr((const void *)gemm_tc_kernel<192, PEpiResidual>, s192) ||
+            !attr((const void *)gemm_tc_kernel<192, PEpiSwiGLU>, s192) ||
+            !attr((const void *)gemm_tc_kernel<128, PEpiQKV>, s128) ||
+            !attr((const void *)gemm_tc_kernel<128, PEpiResidual>, s128) ||
+            !attr((const void *)gemm_tc_kernel<128, PEpiSwiGLU>, s128) ||
             cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)(AttnSmem<128>::TOTAL + 1024)) != cudaSuccess ||
             cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -376,14 +391,22 @@ cudaError_t launch_attn_tc(const Plan &p, const Bufs &b, const PrefillMaps &mp, 
     return cudaGetLastError();
 }
 
-template <class Epi>
-static cudaError_t gemm(const Plan &p, const CUtensorMap *a, const CUtensorMap &w, int T, int N, int K, int *err,
-                        const Epi &epi, cudaStream_t st, LaunchHook *hook, const char *name) {
-    if (hook) hook->before(name);
-    const int tiles = ((T + TC_BM - 1) / TC_BM) * ((N + kPrefillBN - 1) / kPrefillBN);
+template <int BN, class Epi>
+static void launch_gemm(const Plan &p, const CUtensorMap *a, const CUtensorMap &w, int T, int N, int K, int *err,
+                        const Epi &epi, cudaStream_t st) {
+    const int tiles = ((T + TC_BM - 1) / TC_BM) * ((N + BN - 1) / BN);
     const int grid = tiles < p.num_sms ? tiles : p.num_sms;   // persistent: at most one CTA per SM
-    gemm_tc_kernel<kPrefillBN, Epi><<<grid, TC_THREADS, TcTile<kPrefillBN>::SMEM, st>>>(a[0], a[1], a[2], w, T, N, K,
-                                                                                        err, epi);
+    gemm_tc_kernel<BN, Epi><<<grid, TC_THREADS, TcTile<BN>::SMEM, st>>>(a[0], a[1], a[2], w, T, N, K, err, epi);
+}
+
+template <class Epi>
+static cudaError_t gemm(const Plan &p, int bn, const CUtensorMap *a, const CUtensorMap &w, int T, int N, int K,
+                        int *err, const Epi &epi, cudaStream_t st, LaunchHook *hook, const char *name) {
+    if (hook) hook->before(name);
+    if (bn == 128)
+        launch_gemm<128>(p, a, w, T, N, K, err, epi, st);
+    else
+        launch_gemm<192>(p, a, w, T, N, K, err, epi, st);
     if (hook) hook->after(name);
     return cudaGetLastError();
 }
@@ -402,7 +425,7 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.attn_norm, A, p.H, p.cfg.rms_eps);
         PEpiQKV eq = {{{b.Q[0], b.Q[1], b.Q[2]}}, kvl, b.pages, b.rope, p.cfg.qkv_bias ? b.W + lo.bqkv : nullptr, P, p.qdim,
                       p.kvdim, p.d, p.nkv, p.kv_page_elems};
-        if ((e = gemm(p, mp.a, mp.wqkv[l], T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
+        if ((e = gemm(p, mp.bn_qkv, mp.a, mp.wqkv[l], T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
             return e;
         // A5: causal attention over the cache (earlier chunks + this one), tensor cores
         if (hook) hook->before("prefill_attention");
@@ -410,17 +433,17 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         if (hook) hook->after("prefill_attention");
         if (e != cudaSuccess) return e;
         // A6: O projection + residual
-        if ((e = gemm(p, mp.o, mp.wo[l], T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
+        if ((e = gemm(p, mp.bn_o, mp.o, mp.wo[l], T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_o_proj")) != cudaSuccess)
             return e;
         // A7: RMSNorm + gate/up + SwiGLU
         rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.ffn_norm, A, p.H, p.cfg.rms_eps);
         const Terms M = {{b.M[0], b.M[1], b.M[2]}};
-        if ((e = gemm(p, mp.a, mp.wgu[l], T, 2 * p.F, p.H, err, PEpiSwiGLU{M, p.F}, st, hook,
+        if ((e = gemm(p, mp.bn_gu, mp.a, mp.wgu[l], T, 2 * p.F, p.H, err, PEpiSwiGLU{M, p.F}, st, hook,
                       "prefill_gate_up")) != cudaSuccess)
             return e;
         // A8: down projection + residual
-        if ((e = gemm(p, mp.m, mp.wd[l], T, p.H, p.F, err, PEpiResidual{b.X, p.H}, st, hook,
+        if ((e = gemm(p, mp.bn_d, mp.m, mp.wd[l], T, p.H, p.F, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_down")) != cudaSuccess)
             return e;
     }

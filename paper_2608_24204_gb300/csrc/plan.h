@@ -39,7 +39,7 @@ struct Plan {
     size_t kv_elems;
     // workspace (byte offsets)
     size_t ws_ctrl, ws_hist, ws_x, ws_q, ws_o, ws_m, ws_logits, ws_amax, ws_rope,
-        ws_pages, ws_tok, ws_X, ws_fd_part;
+        ws_pages, ws_tok, ws_X, ws_fd_part, ws_mega_bound, ws_mega_time;
     size_t ws_Q[3], ws_A[3], ws_O[3], ws_M[3];   // one buffer per bf16 term
     size_t ws_bytes;
     int num_sms;

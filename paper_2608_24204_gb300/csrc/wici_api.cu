@@ -126,6 +126,8 @@ const char *wici::make_plan(const wici_config *cfg, int num_sms, Plan *p) {
     P.ws_logits = ws(V * 4);
     P.ws_amax = ws((size_t)P.num_sms * sizeof(int2));
     P.ws_fd_part = ws(fd_part_floats(P.nkv, P.group, P.d, P.max_pages) * sizeof(float));
+    P.ws_mega_bound = ws(((size_t)P.num_sms + 1) * sizeof(uint32_t));
+    P.ws_mega_time = ws((size_t)P.num_sms * sizeof(float));
     P.ws_rope = ws((size_t)c.max_tokens * (P.d / 2) * sizeof(float2));
     P.ws_pages = ws((size_t)P.max_pages * 4);
     P.ws_tok = ws(T * 4);
@@ -154,6 +156,8 @@ static Bufs make_bufs(const Plan &p, void *W, void *KV, void *WS) {
     b.logits = (float *)(ws + p.ws_logits);
     b.amax = (int2 *)(ws + p.ws_amax);
     b.fd_part = (float *)(ws + p.ws_fd_part);
+    b.mega_bound = (uint32_t *)(ws + p.ws_mega_bound);
+    b.mega_time = (float *)(ws + p.ws_mega_time);
     b.rope = (float2 *)(ws + p.ws_rope);
     b.pages = (int *)(ws + p.ws_pages);
     b.tok = (int *)(ws + p.ws_tok);
@@ -287,6 +291,17 @@ int wici_create(const wici_config *cfg, void *cuda_stream, void *weight_dev, voi
         // cache slots past the length are read (and weighted by zero) by the
         // tensor-core attention: they must hold finite values from the start
         if ((e = cudaMemsetAsync(c->bufs.KV, 0, p.kv_elems * 2, c->stream)) != cudaSuccess) break;
+        {   // even row shares to start with; the decode kernel refines them step by step
+            std::vector<uint32_t> bound(p.num_sms + 1);
+            for (int i = 0; i <= p.num_sms; ++i)
+                bound[i] = (uint32_t)(((unsigned long long)i << 24) / (unsigned long long)p.num_sms);
+            if ((e = cudaMemcpy(c->bufs.mega_bound, bound.data(), bound.size() * sizeof(uint32_t),
+                                cudaMemcpyHostToDevice)) != cudaSuccess)
+                break;
+            if ((e = cudaMemsetAsync(c->bufs.mega_time, 0, (size_t)p.num_sms * sizeof(float), c->stream)) !=
+                cudaSuccess)
+                break;
+        }
         std::vector<int> pages(p.max_pages);
         for (int i = 0; i < p.max_pages; ++i) pages[i] = i;
         if ((e = cudaMemcpyAsync(c->bufs.pages, pages.data(), pages.size() * 4, cudaMemcpyHostToDevice,
