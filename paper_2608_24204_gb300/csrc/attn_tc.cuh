@@ -5,12 +5,15 @@
 // head g*group + r%group), so each K/V tile serves the whole group.  Keys come
 // from the paged cache in blocks of 64 (four 16-key pages, fetched by 5-D TMA
 // through the page table).  Per block:
-//   S  = (Q_0 + Q_1 + Q_2) K^T    tcgen05.mma, M=128 rows, N=64 keys, fp32 in TMEM
+//   S  = (Q_0 + Q_1) K^T          tcgen05.mma, M=128 rows, N=64 keys, fp32 in TMEM
 //   softmax (one row per thread, read from TMEM): online max/sum, P = exp2(s - m)
-//   O_blk = (P_0 + P_1 + P_2) V   tcgen05.mma, N=d, V read as an MN-major operand
+//   O_blk = (P_0 + P_1) V         tcgen05.mma, N=d, V read as an MN-major operand
 //   O = O * corr + O_blk          in registers
-// Q and P are carried as three bf16 terms like the GEMM activations (fp32
-// precision); K and V are exact bf16.  Warp roles: 0 TMA producer, 1 TMEM owner + MMA issuer, 2..5
+// Q and P are carried as two bf16 terms (hi + lo: 16 significant bits), K and V
+// are exact bf16: the products only meet bf16 K and V, whose own rounding is 2^-9,
+// and the two-term tiles leave room for a three-stage K/V ring (the kernel is
+// bound by the K/V bytes it keeps in flight).  Warp roles: 0 TMA producer,
+// 1 TMEM owner + MMA issuer, 2..5
 // softmax / output (TMEM lane quadrant = warp % 4).  Every wait is bounded.
 #pragma once
 #include <cuda.h>
@@ -24,7 +27,8 @@ namespace wici {
 
 constexpr int AT_ROWS = 128;           // query rows per tile (TMEM lanes)
 constexpr int AT_KEYS = 64;            // keys per block
-constexpr int AT_STAGES = 2;           // K/V ring depth
+constexpr int AT_STAGES = 3;           // K/V ring depth
+constexpr int AT_TERMS = 2;            // bf16 terms of the Q and P operands
 constexpr int AT_THREADS = 192;
 constexpr uint32_t AT_TMEM_COLS = 256; // S: [0, 64), O block: [128, 128 + d)
 
@@ -38,9 +42,9 @@ struct AttnSmem {
     static constexpr uint32_t KV_BYTES = AT_KEYS * D * 2;                // K (or V) of a block
     static constexpr uint32_t P_BYTES = AT_ROWS * AT_KEYS * 2;           // one term
     static constexpr uint32_t OFF_Q = 0;                                 // [term]
-    static constexpr uint32_t OFF_KV = kTerms * Q_BYTES;                 // [stage][K | V]
+    static constexpr uint32_t OFF_KV = AT_TERMS * Q_BYTES;               // [stage][K | V]
     static constexpr uint32_t OFF_P = OFF_KV + AT_STAGES * 2 * KV_BYTES; // [term]
-    static constexpr uint32_t TOTAL = OFF_P + kTerms * P_BYTES;
+    static constexpr uint32_t TOTAL = OFF_P + AT_TERMS * P_BYTES;
 };
 
 // K-major, 128-byte swizzle, 8-row groups 1024 B apart (Q, K and P operands)
@@ -100,7 +104,7 @@ struct AttnArgs {
 template <int D>
 __global__ void __launch_bounds__(AT_THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap map_q0, const __grid_constant__ CUtensorMap map_q1,
-                   const __grid_constant__ CUtensorMap map_q2, const __grid_constant__ CUtensorMap map_kv,
+                   const __grid_constant__ CUtensorMap map_kv,
                    const AttnArgs a) {
     using L = AttnSmem<D>;
     extern __shared__ uint8_t smem_raw[];
@@ -145,12 +149,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     if (warp == 0) {
         if (lane == 0) {  // ----------------------------------------------- TMA producer
             const uint32_t qb = smem_u32(&q_full);
-            mbar_arrive_expect_tx(qb, (uint32_t)kTerms * L::DCH * q_bytes_box);
+            mbar_arrive_expect_tx(qb, (uint32_t)AT_TERMS * L::DCH * q_bytes_box);
             for (int c = 0; c < L::DCH; ++c) {
                 tma_load_3d(base + L::OFF_Q + c * AT_ROWS * 128, &map_q0, c * 64, g * a.group, t0, qb);
                 tma_load_3d(base + L::OFF_Q + L::Q_BYTES + c * AT_ROWS * 128, &map_q1, c * 64, g * a.group, t0, qb);
-                tma_load_3d(base + L::OFF_Q + 2 * L::Q_BYTES + c * AT_ROWS * 128, &map_q2, c * 64, g * a.group, t0,
-                            qb);
             }
             int issued = 0;
             for (int j = 0; j < nb; ++j) {
@@ -193,7 +195,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                     const uint32_t koff = (uint32_t)(k / 4) * (AT_KEYS * 128) + 32u * (k % 4);
                     const uint64_t bd = at_desc_k(kb + koff);
 #pragma unroll
-                    for (int t = 0; t < kTerms; ++t)
+                    for (int t = 0; t < AT_TERMS; ++t)
                         tc_mma(tm_s, at_desc_k(base + L::OFF_Q + t * L::Q_BYTES + off), bd, idesc_s, (k | t) != 0);
                 }
                 tc_commit(smem_u32(&s_full));
@@ -210,7 +212,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                     // 16 keys = two 8-key groups of V rows; P columns 16k..16k+15
                     const uint64_t vd = at_desc_mn(vb + 2048u * k, AT_KEYS * 128);
 #pragma unroll
-                    for (int t = 0; t < kTerms; ++t)
+                    for (int t = 0; t < AT_TERMS; ++t)
                         tc_mma(tm_o, at_desc_k(base + L::OFF_P + t * L::P_BYTES + 32u * k), vd, idesc_o, (k | t) != 0);
                 }
                 tc_commit(smem_u32(&o_full));
@@ -249,27 +251,24 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             const float msafe = mn == -INFINITY ? 0.f : mn;   // rows with nothing visible yet
             const float corr = exp2f(m - msafe);
             float ps = 0.f;
-            // P row r as three bf16 terms, 128-byte swizzled rows (16-byte piece i at i ^ (r % 8))
+            // P row r as two bf16 terms, 128-byte swizzled rows (16-byte piece i at i ^ (r % 8))
             uint8_t *prow = pbase + r * 128;
 #pragma unroll
             for (int piece = 0; piece < AT_KEYS / 8; ++piece) {
-                uint32_t w0[4], w1[4], w2[4];
+                uint32_t w0[4], w1[4];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     const float p0 = exp2f(sv[piece * 8 + 2 * e] - msafe);
                     const float p1 = exp2f(sv[piece * 8 + 2 * e + 1] - msafe);
                     ps += p0 + p1;
-                    uint16_t a0, a1, a2, b0, b1, b2;
-                    split_bf16x3(p0, a0, a1, a2);
-                    split_bf16x3(p1, b0, b1, b2);
+                    const uint16_t a0 = f32_to_bf16(p0), b0 = f32_to_bf16(p1);
+                    const uint16_t a1 = f32_to_bf16(p0 - bf16_to_f32(a0)), b1 = f32_to_bf16(p1 - bf16_to_f32(b0));
                     w0[e] = (uint32_t)a0 | ((uint32_t)b0 << 16);
                     w1[e] = (uint32_t)a1 | ((uint32_t)b1 << 16);
-                    w2[e] = (uint32_t)a2 | ((uint32_t)b2 << 16);
                 }
                 const int sp = (piece ^ (r & 7)) * 16;
                 *reinterpret_cast<uint4 *>(prow + sp) = make_uint4(w0[0], w0[1], w0[2], w0[3]);
                 *reinterpret_cast<uint4 *>(prow + L::P_BYTES + sp) = make_uint4(w1[0], w1[1], w1[2], w1[3]);
-                *reinterpret_cast<uint4 *>(prow + 2 * L::P_BYTES + sp) = make_uint4(w2[0], w2[1], w2[2], w2[3]);
             }
             l = l * corr + ps;
             m = mn;

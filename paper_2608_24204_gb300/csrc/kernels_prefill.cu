@@ -383,10 +383,10 @@ cudaError_t launch_attn_tc(const Plan &p, const Bufs &b, const PrefillMaps &mp, 
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)p.d);
     dim3 grid((T + a.tpt - 1) / a.tpt, p.nkv);
     if (p.d == 128)
-        attn_tc_kernel<128><<<grid, AT_THREADS, AttnSmem<128>::TOTAL + 1024, st>>>(mp.q[0], mp.q[1], mp.q[2], mp.kv,
+        attn_tc_kernel<128><<<grid, AT_THREADS, AttnSmem<128>::TOTAL + 1024, st>>>(mp.q[0], mp.q[1], mp.kv,
                                                                                   a);
     else
-        attn_tc_kernel<64><<<grid, AT_THREADS, AttnSmem<64>::TOTAL + 1024, st>>>(mp.q[0], mp.q[1], mp.q[2], mp.kv,
+        attn_tc_kernel<64><<<grid, AT_THREADS, AttnSmem<64>::TOTAL + 1024, st>>>(mp.q[0], mp.q[1], mp.kv,
                                                                                 a);
     return cudaGetLastError();
 }
