@@ -37,7 +37,7 @@
 namespace wici {
 
 constexpr int TC_BM = 128, TC_BK = 64, TC_THREADS = 320, TC_EPI_WARPS = 8;
-constexpr int TC_GROUP = 2;                                             // k-blocks per TMEM accumulation
+constexpr int TC_GROUP = 4;                                             // k-blocks per TMEM accumulation
 constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;                      // 16 KB per term
 constexpr uint32_t TC_TMEM_COLS = 512;                                  // two accumulator buffers
 constexpr size_t TC_SMEM_BUDGET = 216 * 1024;                           // ring bytes
