@@ -139,7 +139,10 @@ const char *wici_last_error(const wici_ctx *ctx);
  * bracketed by CUDA events on the context's stream (for roofline accounting).
  * For each kernel kind i < *n_kinds: names[i] (static string), launches[i] and
  * total_ms[i].  Arrays have room for `cap` entries.  Advances kv_len by n_steps
- * like wici_decode. */
+ * like wici_decode.  Where the step runs as one persistent kernel there is a
+ * single kind, "decode_step"; otherwise one kind per layer operation
+ * ("qkv_rope_kvappend", "flash_decode", "o_proj_residual", "gate_up_swiglu",
+ * "down_residual") plus "lm_head_argmax". */
 int wici_profile_decode(wici_ctx *ctx, int32_t n_steps, const char **names, int32_t *launches,
                         double *total_ms, int32_t cap, int32_t *n_kinds);
 

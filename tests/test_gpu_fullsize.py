@@ -39,3 +39,9 @@ def test_llama3_8b_shape_bench_launch_configuration():
 def test_llama32_1b_shape_full_prompt():
     stats = _full(gen.LLAMA_1B, decode_steps=8)
     assert len(stats["max_abs"]) == 9
+
+
+def test_qwen25_14b_shape_full_prompt():
+    # the deepest config: 48 layers, a 2048-token prompt, then one decode step
+    stats = _full(gen.QWEN_14B, decode_steps=1)
+    assert len(stats["max_abs"]) == 2
