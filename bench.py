@@ -142,6 +142,22 @@ class ClockSampler:
                 "reasons": sorted(reasons)}
 
 
+def max_over_ranks(values, world: int, device: str = "cuda"):
+    """Element-wise maximum of `values` over all ranks (the slowest rank's times)."""
+    import torch
+    t = torch.tensor(list(values), dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t]
+
+
+def job_tokens_per_s(world: int, local_tokens: int, slowest_s: float) -> float:
+    """Whole-job decode rate: every replica decodes `local_tokens`; the job ends
+    with the slowest one."""
+    return world * local_tokens / slowest_s
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -258,11 +274,8 @@ def run_ours(args):
     dec = [e[1].elapsed_time(e[2]) for e in evs]
     dec_s = sum(dec) / 1000.0
     local_tok = args.steps * DECODE
-    t_max = torch.tensor([dec_s, total_ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        torch.distributed.all_reduce(t_max, op=torch.distributed.ReduceOp.MAX)
-    dec_s_max, total_ms_max = float(t_max[0]), float(t_max[1])
-    value = world * local_tok / dec_s_max
+    dec_s_max, total_ms_max = max_over_ranks([dec_s, total_ms], world)
+    value = job_tokens_per_s(world, local_tok, dec_s_max)
 
     # bytes per decoded token (weights + KV of the context), averaged over the 256 steps
     bytes_tok = sum(gen.decode_bytes_per_token(CFG, PROMPT + i) for i in range(1, DECODE + 1)) / DECODE
