@@ -26,6 +26,8 @@ and listed with the same wording in the design notes:
     a diagnostic that isolates operand rounding from errors.
   * QKV bias (Qwen2.5 shape) is added before RoPE; no other biases.
   * Greedy token = argmax of the logits, lowest index on an exact tie.
+  * Optional `q8_weights`: matrices in the 8-bit block format (oracle/q8.py)
+    replace the bf16 tensors of the same name.
 
 Parity pins for every function are in `tests/test_oracle_pins.py`.
 """
@@ -139,9 +141,12 @@ class OracleModel:
     """
 
     def __init__(self, cfg, weights: dict, prefill_act_bf16: bool = False,
-                 max_tokens: int | None = None, cache_bytes: float = 6e9):
+                 max_tokens: int | None = None, cache_bytes: float = 6e9, q8_weights: dict | None = None):
         self.cfg = cfg
         self.w = weights
+        # matrices given in the 8-bit block format ({name: (codes, scales)}) take
+        # the place of the bf16 tensors of the same name
+        self.q8 = q8_weights or {}
         self.prefill_act_bf16 = prefill_act_bf16
         self._act_round = round_bf16
         self.max_tokens = max_tokens or cfg.total_tokens
@@ -159,7 +164,11 @@ class OracleModel:
     def W(self, name: str) -> np.ndarray:
         if self._cache is not None and name in self._cache:
             return self._cache[name]
-        m = bf16_bits_to_f64(self.w[name])
+        if name in self.q8:
+            from .q8 import q8_dequantize
+            m = q8_dequantize(*self.q8[name])
+        else:
+            m = bf16_bits_to_f64(self.w[name])
         if self._cache is not None:
             self._cache[name] = m
         return m

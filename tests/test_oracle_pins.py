@@ -240,11 +240,14 @@ def test_incremental_decode_equals_full_causal_recompute():
     np.testing.assert_allclose(got, want, rtol=1e-9, atol=1e-11)
 
 
-def _torch_restatement(cfg, w, tokens):
+def _torch_restatement(cfg, w, tokens, mats=None):
     """The whole forward, written independently with torch library ops (fp64):
     F.rms_norm, complex-number RoPE, F.linear (with the QKV bias when present),
-    F.scaled_dot_product_attention on repeated KV heads, F.silu."""
+    F.scaled_dot_product_attention on repeated KV heads, F.silu.  `mats`, when
+    given, supplies fp64 torch matrices that take the place of bf16 tensors."""
     def W(n):
+        if mats is not None and n in mats:
+            return mats[n]
         return torch.from_numpy((w[n].astype(np.uint32) << 16).view(np.float32)).double()
 
     def B(n):
