@@ -87,10 +87,14 @@ typedef struct wici_tensor {
 } wici_tensor;
 
 /* Sizes of the three caller-owned device buffers for `cfg`.  WICI_E_ARG on an
- * invalid configuration. */
+ * invalid configuration.  (Sec. 3.2, context management: the application's
+ * own memory on the server's native CUDA context holds the model; here the
+ * caller allocates it, the library only lays it out.) */
 int wici_get_sizes(const wici_config *cfg, wici_sizes *out);
 
-/* Create a context on the current CUDA device.  `cuda_stream` (a cudaStream_t,
+/* Create a context on the current CUDA device (Sec. 3.2: each client is served
+ * by its own server thread on the native CUDA context; one wici_ctx per
+ * client thread).  `cuda_stream` (a cudaStream_t,
  * may be NULL for the legacy stream) orders every launch of this context; the
  * three buffers must be at least wici_get_sizes() bytes and 256-byte aligned.
  * The KV page table starts as the identity.  *out receives the context. */
@@ -113,29 +117,36 @@ int wici_prefill(wici_ctx *ctx, const int32_t *tokens, int32_t n, float *logits_
 /* One decode step: feed `token_in` (>= 0), or the last greedy token when
  * token_in < 0, at position kv_len; kv_len += 1.  Outputs as for wici_prefill.
  * Runs the captured CUDA graph of the whole step.  WICI_E_STATE before the
- * first prefill. */
+ * first prefill.  (T_Local of Eq. 1, Sec. 3.3: the GPU time of one generated
+ * token; Sec. 4.2.2, trace replay: every token repeats the same computation
+ * with only the input token changing, so one recorded graph is replayed.) */
 int wici_decode_step(wici_ctx *ctx, int32_t token_in, float *logits_out, int32_t *token_out);
 
-/* `n_steps` greedy decode steps back to back on the device (each step feeds
+/* Sec. 4.2.2 (trace replay without a round trip per token):
+ * `n_steps` greedy decode steps back to back on the device (each step feeds
  * the previous step's argmax; the first feeds token_in, or the last greedy
  * token if token_in < 0).  tokens_out (nullable, host int32[n_steps]) receives
  * the generated tokens. */
 int wici_decode(wici_ctx *ctx, int32_t n_steps, int32_t token_in, int32_t *tokens_out);
 
-/* Forget the cached tokens (kv_len := 0); weights stay loaded. */
+/* Forget the cached tokens (kv_len := 0); weights stay loaded.  (Sec. 5.1:
+ * every evaluated sample is a new request on the already loaded model.) */
 int wici_reset(wici_ctx *ctx);
 
 /* Replace the logical->physical KV page map (host int32[n], n = max_tokens/16
- * rounded up, a permutation of 0..n-1).  Only valid when kv_len == 0. */
+ * rounded up, a permutation of 0..n-1).  Only valid when kv_len == 0.  The
+ * paper has no counterpart: the paged cache is this library's layout. */
 int wici_set_page_table(wici_ctx *ctx, const int32_t *pages, int32_t n);
 
-/* Number of cached positions, or a negative status. */
+/* Number of cached positions, or a negative status (bookkeeping; no paper
+ * counterpart). */
 int32_t wici_kv_len(const wici_ctx *ctx);
 
 /* Message of the last error on ctx (or of this thread when ctx is NULL). */
 const char *wici_last_error(const wici_ctx *ctx);
 
-/* Per-kernel timing of `n_steps` decode steps run as individual launches, each
+/* Measurement of T_Local (Eq. 1, Sec. 3.3) per kernel.
+ * Per-kernel timing of `n_steps` decode steps run as individual launches, each
  * bracketed by CUDA events on the context's stream (for roofline accounting).
  * For each kernel kind i < *n_kinds: names[i] (static string), launches[i] and
  * total_ms[i].  Arrays have room for `cap` entries.  Advances kv_len by n_steps
@@ -146,7 +157,8 @@ const char *wici_last_error(const wici_ctx *ctx);
 int wici_profile_decode(wici_ctx *ctx, int32_t n_steps, const char **names, int32_t *launches,
                         double *total_ms, int32_t cap, int32_t *n_kinds);
 
-/* Self-test of the bounded device wait: launches one CTA that waits on an
+/* Failure detection (no paper counterpart).
+ * Self-test of the bounded device wait: launches one CTA that waits on an
  * mbarrier nobody arrives at, giving up after `limit_ns` nanoseconds.  Returns
  * WICI_E_TIMEOUT when the wait gave up as designed (the expected result). */
 int wici_check_bounded_wait(void *cuda_stream, int64_t limit_ns);
@@ -171,6 +183,10 @@ int wici_check_bounded_wait(void *cuda_stream, int64_t limit_ns);
  *   token_dev      device int32 [1], receives the argmax (lowest index on ties)
  * All work is enqueued on cuda_stream (a cudaStream_t, NULL for the legacy
  * stream); the call does not synchronise.  The device is the current one.
+ * The call returns before the GPU has run, so a device-side failure cannot
+ * reach its return code: if a bounded wait inside the kernel gives up,
+ * *token_dev receives -1 instead of a vocabulary index, and the logits are
+ * then incomplete.  Check the token for -1 before using either output.
  * Limits: hidden a multiple of 8 in [8, 16384]; vocab >= 1; the current GPU
  * may have at most 1024 SMs (one scratch partial per CTA); anything else
  * returns WICI_E_ARG with the reason in wici_last_error(NULL).
@@ -184,7 +200,8 @@ int wici_lm_head_argmax_noalloc(void *cuda_stream, const void *lm_head_dev, cons
                                 const float *x_dev, int32_t hidden, int32_t vocab, float rms_eps,
                                 float *logits_dev, int32_t *token_dev);
 
-/* Destroy the context (frees only what the library allocated). */
+/* Destroy the context (frees only what the library allocated).  (Sec. 5.4,
+ * multiple clients: a client that disconnects releases its server thread.) */
 void wici_destroy(wici_ctx *ctx);
 
 #ifdef __cplusplus

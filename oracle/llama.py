@@ -176,8 +176,9 @@ class OracleModel:
     def _vec(self, name: str) -> np.ndarray:
         return self.W(name).reshape(-1)
 
-    def forward(self, tokens, round_act: bool = False) -> np.ndarray:
-        """Run tokens at positions kv_len..kv_len+T-1; return logits [V] of the last one."""
+    def forward(self, tokens, round_act: bool = False, all_rows: bool = False) -> np.ndarray:
+        """Run tokens at positions kv_len..kv_len+T-1; return logits [V] of the last
+        one, or with `all_rows` the logits [T, V] after every one of them."""
         cfg = self.cfg
         tokens = np.asarray(tokens, np.int64).reshape(-1)
         T, P = len(tokens), self.kv_len
@@ -212,8 +213,10 @@ class OracleModel:
             m = silu(h2 @ self.W(p + "wg").T) * (h2 @ self.W(p + "wu").T)
             x = x + rnd(m) @ self.W(p + "wd").T
         self.kv_len = P + T
-        hf = rmsnorm(x[-1], self._vec("final_norm"), cfg.rms_eps)
         lm = "embed" if cfg.tied_embeddings else "lm_head"
+        if all_rows:
+            return rmsnorm(x, self._vec("final_norm"), cfg.rms_eps) @ self.W(lm).T
+        hf = rmsnorm(x[-1], self._vec("final_norm"), cfg.rms_eps)
         return self.W(lm) @ hf
 
     def prefill(self, tokens):
@@ -223,6 +226,14 @@ class OracleModel:
     def decode(self, token: int):
         logits = self.forward([token], round_act=False)
         return logits, greedy(logits)
+
+    def decode_forced(self, tokens) -> np.ndarray:
+        """Decode steps fed a known token sequence (teacher forcing), taken as one
+        pass: appends the tokens and returns [T, V], whose row t is what
+        decode(tokens[t]) would return at that point.  A causal pass over known
+        tokens is the same computation as feeding them one at a time (the KV
+        cache only ever holds earlier positions)."""
+        return self.forward(tokens, round_act=False, all_rows=True)
 
 
 def run_workload(cfg, weights, prompts, decode_steps: int, **kw):

@@ -64,6 +64,12 @@ int setup_device(int dev, NoAllocScratch **out, int *nsm) {
     return WICI_OK;
 }
 
+// Hands the token to the caller, or -1 when a bounded wait inside the LM-head
+// kernel gave up (its logits are then incomplete and its token meaningless).
+__global__ void noalloc_publish_token(const int *ctrl, int32_t *token) {
+    token[0] = ctrl[CTRL_ERR] != 0 ? -1 : ctrl[CTRL_TOKEN];
+}
+
 }  // namespace
 
 extern "C" int wici_lm_head_argmax_noalloc(void *cuda_stream, const void *lm_head_dev, const void *norm_gain_dev,
@@ -86,15 +92,14 @@ extern "C" int wici_lm_head_argmax_noalloc(void *cuda_stream, const void *lm_hea
     if (grid > kNoAllocMaxCtas)
         return fail(WICI_E_ARG, "needs %d argmax partials, the fixed scratch holds %d", grid, kNoAllocMaxCtas);
     cudaStream_t st = (cudaStream_t)cuda_stream;
-    // the ticket, position and token words must start at zero on every call
+    // the ticket, position, token and error words must start at zero on every call
     if ((e = cudaMemsetAsync(sc->ctrl, 0, sizeof sc->ctrl, st)) != cudaSuccess)
         return fail(WICI_E_CUDA, "clear scratch: %s", cudaGetErrorString(e));
     if ((e = enqueue_lm_head_argmax_raw((const uint16_t *)lm_head_dev, (const uint16_t *)norm_gain_dev, x_dev,
                                         hidden, vocab, rms_eps, logits_dev, sc->ctrl, sc->partials, sc->hist, grid,
                                         st)) != cudaSuccess)
         return fail(WICI_E_CUDA, "launch: %s", cudaGetErrorString(e));
-    if ((e = cudaMemcpyAsync(token_dev, sc->ctrl + CTRL_TOKEN, sizeof(int32_t), cudaMemcpyDeviceToDevice, st)) !=
-        cudaSuccess)
-        return fail(WICI_E_CUDA, "token copy: %s", cudaGetErrorString(e));
+    noalloc_publish_token<<<1, 1, 0, st>>>(sc->ctrl, token_dev);
+    if ((e = cudaGetLastError()) != cudaSuccess) return fail(WICI_E_CUDA, "token publish: %s", cudaGetErrorString(e));
     return WICI_OK;
 }

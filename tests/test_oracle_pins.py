@@ -240,6 +240,29 @@ def test_incremental_decode_equals_full_causal_recompute():
     np.testing.assert_allclose(got, want, rtol=1e-9, atol=1e-11)
 
 
+def test_forced_decode_rows_equal_step_by_step_decode():
+    # decode_forced feeds a known token sequence in one causal pass; each row must
+    # be the logits that feeding the tokens one step at a time gives
+    cfg = gen.TINY
+    w = _tiny_weights(cfg)
+    prompt = gen.make_prompt(cfg, 12, seed=1)
+    forced = gen.make_prompt(cfg, 6, seed=9)
+    step = oracle.OracleModel(cfg, w, max_tokens=32)
+    step.prefill(prompt)
+    want = [step.decode(int(t)) for t in forced]
+    one = oracle.OracleModel(cfg, w, max_tokens=32)
+    first, _ = one.prefill(prompt)
+    rows = one.decode_forced(forced)
+    assert rows.shape == (len(forced), cfg.vocab) and one.kv_len == step.kv_len
+    for r, (logits, tok) in zip(rows, want):
+        np.testing.assert_allclose(r, logits, rtol=1e-9, atol=1e-11)
+        assert oracle.greedy(r) == tok
+    # the last row of an all-rows pass is the ordinary last-position result
+    a = oracle.OracleModel(cfg, w, max_tokens=32)
+    b = oracle.OracleModel(cfg, w, max_tokens=32)
+    np.testing.assert_allclose(a.forward(prompt, all_rows=True)[-1], b.forward(prompt), rtol=1e-12, atol=1e-13)
+
+
 def _torch_restatement(cfg, w, tokens, mats=None):
     """The whole forward, written independently with torch library ops (fp64):
     F.rms_norm, complex-number RoPE, F.linear (with the QKV bias when present),
