@@ -9,9 +9,12 @@ flush is needed between steps.
 
 Beside the decode roofline (`roofline`, the dominant kernel) the line carries
 `prefill_roofline` (the request's prefill FLOPs / TTFT against the bf16 tensor
-peak) and `agentic`: the agentic long-context workload at the same shape
+peak), `agentic`: the agentic long-context workload at the same shape
 (4 turns of a 2048-token chunk plus 64 decode steps, 8448 cached), timed after
-the K requests, with its four chunk prefills in aggregate against the bf16 peak.
+the K requests, with its four chunk prefills in aggregate against the bf16 peak,
+`multi_tenant`: a 1B-shaped and the 8B-shaped model decoding at the same
+time on SM shares of one GPU, per-tenant tokens/s, and `q8`: the 8B request
+with its per-layer matrices in the 8-bit block format.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -236,6 +239,112 @@ def measure_agentic(weights, WiciModel, torch, pk, runs: int = 3):
             "runs": runs}
 
 
+def measure_q8(weights_8b, WiciModel, torch, pk, runs: int = 3):
+    """The Llama-3-8B-shaped request with the seven per-layer matrices in the
+    8-bit block format (int8 codes + one fp16 scale per 32; the embedding, norms
+    and LM head stay bf16): 1024-token prompt, then 256 greedy decode steps.
+    Decode tokens/s and bytes/s over the format's algorithmic bytes per token,
+    the decode kernel's own launch time (CUDA events), and the TTFT."""
+    from gen import q8 as gq
+    from paper_2608_24204_gb300 import wici
+    q8w = gq.make_q8_weights(CFG)
+    model = WiciModel(CFG, max_tokens=PROMPT + DECODE + 16, max_chunk=PROMPT, q8=True).load(weights_8b, q8w)
+    del q8w
+    prompt = gen.make_prompt(CFG, PROMPT, seed=1)
+    st = model.stream
+    ttft, dec = [], []
+    for r in range(runs + 1):
+        model.reset()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        ev[0].record(st)
+        model.prefill(prompt)
+        ev[1].record(st)
+        model.decode(DECODE)
+        ev[2].record(st)
+        torch.cuda.synchronize()
+        if r > 0:
+            ttft.append(ev[0].elapsed_time(ev[1]))
+            dec.append(ev[1].elapsed_time(ev[2]))
+    model.reset()
+    model.prefill(prompt)
+    n_prof = 8
+    prof = wici.wici_profile_decode(model.ctx, n_prof)
+    model.close()
+    n_k, ms_k = prof["decode_step"]
+    unit_bytes = sum(gen.decode_bytes_per_token(CFG, PROMPT + i, q8=True) for i in range(1, n_prof + 1)) / n_prof
+    k_gbs = unit_bytes / (ms_k / n_k / 1000.0) / 1e9
+    bytes_tok = sum(gen.decode_bytes_per_token(CFG, PROMPT + i, q8=True) for i in range(1, DECODE + 1)) / DECODE
+    dec_s = statistics.median(dec) / 1000.0
+    return {"workload": f"{CFG.name} in the 8-bit block format: prompt {PROMPT}, {DECODE} greedy decode steps",
+            "decode_tok_s": DECODE / dec_s, "bytes_per_token": bytes_tok,
+            "decode_gbs": bytes_tok * DECODE / dec_s / 1e9,
+            "decode_frac_of_measured_hbm": bytes_tok * DECODE / dec_s / 1e9 / pk["hbm_gbs"],
+            "decode_frac_of_8tbs": bytes_tok * DECODE / dec_s / 1e9 / NOMINAL_HBM_GBS,
+            "roofline": {"bound": "hbm", "kernel": "decode_step (8-bit)", "achieved": k_gbs, "peak": pk["hbm_gbs"],
+                         "unit": "GB/s", "frac": k_gbs / pk["hbm_gbs"], "bytes_per_launch": unit_bytes,
+                         "avg_launch_us": ms_k / n_k * 1000.0},
+            "ttft_ms": statistics.median(ttft), "runs": runs}
+
+
+def measure_multi_tenant(weights_8b, WiciModel, torch, steps: int = 256):
+    """Two tenants on one GPU, as in the paper's two-client microbenchmark: a
+    Llama-3.2-1B-shaped model (512-token prompt) and the Llama-3-8B-shaped one
+    (1024-token prompt), each with an SM share (a quarter and the rest) so that
+    both persistent decode grids are resident at once, each on its own stream
+    (the small model's at the higher priority).  Decode tokens/s of each
+    tenant alone on its share, then with both decoding at the same time from
+    two host threads; CUDA events on each tenant's stream."""
+    import threading
+    nsm = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    shares = {"small": nsm // 4, "large": nsm - nsm // 4}
+    cfgs = {"small": gen.LLAMA_1B, "large": gen.LLAMA_8B}
+    prompts = {k: gen.make_prompt(c, c.prompt_len, seed=1) for k, c in cfgs.items()}
+    models = {}
+    for k, c in cfgs.items():
+        w = weights_8b if k == "large" else gen.make_weights(c)
+        st = torch.cuda.Stream(priority=-1 if k == "small" else 0)
+        models[k] = WiciModel(c, max_tokens=c.prompt_len + steps + 16, max_chunk=c.prompt_len, stream=st,
+                              max_sms=shares[k]).load(w)
+
+    def timed_decode(k, out):
+        m = models[k]
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(m.stream)
+        m.decode(steps)
+        e1.record(m.stream)
+        e1.synchronize()
+        out[k] = steps / (e0.elapsed_time(e1) / 1000.0)
+
+    def prime():
+        for k, m in models.items():
+            m.reset()
+            m.prefill(prompts[k])
+        torch.cuda.synchronize()
+
+    prime()
+    for k in models:               # warm-up (graph capture, row shares)
+        timed_decode(k, {})
+    alone = {}
+    for k in models:
+        prime()
+        timed_decode(k, alone)
+    prime()
+    together = {}
+    th = [threading.Thread(target=timed_decode, args=(k, together)) for k in models]
+    for t in th:
+        t.start()
+    for t in th:
+        t.join()
+    for m in models.values():
+        m.close()
+    return {"workload": f"tenant small: {gen.LLAMA_1B.name} (prompt {gen.LLAMA_1B.prompt_len}), "
+                        f"tenant large: {gen.LLAMA_8B.name} (prompt {gen.LLAMA_8B.prompt_len}); "
+                        f"{steps} greedy decode steps each",
+            "sm_share": shares, "stream_priority": {"small": -1, "large": 0},
+            "tok_s_alone_on_share": alone, "tok_s_together": together,
+            "unit": "tok/s"}
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -393,11 +502,13 @@ def run_ours(args):
                         "flops_per_prefill": pf_flops, "ttft_ms": ttft_med, "peak_source": pk["source"],
                         "what": f"algorithmic FLOPs of the {PROMPT}-token prefill / TTFT (CUDA events)"}
 
-    agentic = None
+    agentic = tenants = q8 = None
     if not args.no_agentic and CFG.n_layers == gen.LLAMA_8B.n_layers:
         model.close()
         model = None
         agentic = measure_agentic(weights, WiciModel, torch, pk)
+        tenants = measure_multi_tenant(weights, WiciModel, torch)
+        q8 = measure_q8(weights, WiciModel, torch, pk)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -423,6 +534,7 @@ def run_ours(args):
             "bytes_per_token": bytes_tok,
             "prefill_tflops": pf_tf,
             "roofline": roofline, "prefill_roofline": prefill_roofline, "agentic": agentic,
+            "multi_tenant": tenants, "q8": q8,
             "kernels": kernel_share, "cpu_baseline": cpu,
             "e2e": {"value": e2e_val, "unit": "tok/s", "h2d_bytes_per_step": PROMPT * 4,
                     "d2h_bytes_per_step": (DECODE + 1) * 4, "ttft_ms": statistics.median(e2e_ttft),
@@ -447,7 +559,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-agentic", action="store_true", help="skip the agentic 4 x 2048 prefill measurement")
+    ap.add_argument("--no-agentic", action="store_true",
+                    help="skip the agentic, two-tenant and 8-bit-format measurements")
     ap.add_argument("--quick", action="store_true", help="profiling run: timed requests only")
     ap.add_argument("--decode-steps", type=int, default=0, help="profiling run: decode steps per request")
     ap.add_argument("--layers", type=int, default=0, help="profiling run: fewer layers (small ncu case)")

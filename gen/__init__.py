@@ -10,7 +10,7 @@ import threading
 
 import numpy as np
 
-from .configs import (CONFIGS, LLAMA_1B, LLAMA_8B, LLAMA_8B_AGENTIC, QWEN_14B, TINY,
+from .configs import (CONFIGS, LLAMA_1B, LLAMA_8B, LLAMA_8B_AGENTIC, QWEN3_8B, QWEN_14B, TINY,
                       ModelConfig, decode_bytes_per_token, prefill_flops, tensor_specs)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -20,6 +20,7 @@ _lock = threading.Lock()
 _lib = None
 
 PROMPT_TAG = 0x7FFFFFFF
+GAIN_STD = 0.25   # per-head q/k norm gains: 1 + 0.25 N(0, 1), rounded to bf16
 
 
 def build(force: bool = False) -> str:
@@ -46,6 +47,7 @@ def _load():
             lib.wicigen_normal_f64.argtypes = [u64, u64, u64, u64, p]
             lib.wicigen_tokens.argtypes = [u64, u64, u64, u64, p]
             lib.wicigen_fill_bf16.argtypes = [ctypes.c_float, u64, p]
+            lib.wicigen_gain_bf16.argtypes = [u64, u64, dbl, u64, u64, p]
             _lib = lib
     return _lib
 
@@ -78,6 +80,8 @@ def make_tensor(cfg: ModelConfig, name: str, out: np.ndarray | None = None) -> n
     lib = _load()
     if kind == "ones":
         lib.wicigen_fill_bf16(1.0, out.size, out.ctypes.data)
+    elif kind == "gain":
+        lib.wicigen_gain_bf16(cfg.weight_seed, tag, GAIN_STD, 0, out.size, out.ctypes.data)
     else:
         lib.wicigen_normal_bf16(cfg.weight_seed, tag, cfg.weight_std, 0, out.size, out.ctypes.data)
     return out
@@ -97,6 +101,6 @@ def make_prompt(cfg: ModelConfig, n: int, seed: int = 1) -> np.ndarray:
     return out
 
 
-__all__ = ["CONFIGS", "TINY", "LLAMA_1B", "LLAMA_8B", "LLAMA_8B_AGENTIC", "QWEN_14B",
+__all__ = ["CONFIGS", "TINY", "LLAMA_1B", "LLAMA_8B", "LLAMA_8B_AGENTIC", "QWEN_14B", "QWEN3_8B",
            "ModelConfig", "tensor_specs", "decode_bytes_per_token", "prefill_flops",
            "make_tensor", "make_weights", "make_prompt", "normal_f64", "draw", "stream", "build"]

@@ -25,6 +25,7 @@ class ModelConfig:
     rms_eps: float = 1e-5
     tied_embeddings: bool = False
     qkv_bias: bool = False
+    qk_norm: bool = False          # Qwen3 block: per-head RMSNorm of q and k before RoPE
     weight_std: float = 0.02
     weight_seed: int = 0
     # workload: `turns` rounds of (prompt_len-token chunk, then decode_steps greedy tokens)
@@ -76,11 +77,19 @@ QWEN_14B = ModelConfig(
     ffn_dim=13824, vocab=152064, rope_theta=1000000.0, rms_eps=1e-6, qkv_bias=True,
     prompt_len=2048, decode_steps=256)
 
-CONFIGS = {c.name: c for c in (TINY, LLAMA_1B, LLAMA_8B, LLAMA_8B_AGENTIC, QWEN_14B)}
+# The paper's headline model family (Qwen3, Tab. 1) at the 8B shape: the Llama
+# block plus a per-head RMSNorm of q and k before RoPE, no QKV bias, untied.
+QWEN3_8B = ModelConfig(
+    name="qwen3-8b", n_layers=36, hidden=4096, n_q_heads=32, n_kv_heads=8, head_dim=128,
+    ffn_dim=12288, vocab=151936, rope_theta=1000000.0, rms_eps=1e-6, qk_norm=True,
+    prompt_len=1024, decode_steps=256)
+
+CONFIGS = {c.name: c for c in (TINY, LLAMA_1B, LLAMA_8B, LLAMA_8B_AGENTIC, QWEN_14B, QWEN3_8B)}
 
 
 def tensor_specs(cfg: ModelConfig):
-    """Canonical tensor list: (name, (rows, cols), kind) with kind 'normal' or 'ones'.
+    """Canonical tensor list: (name, (rows, cols), kind) with kind 'normal', 'ones'
+    or 'gain' (1 + 0.25 N(0, 1): the per-head q/k norm gains, not all one).
 
     The position of a tensor in this list is its generator tag.  All matrices
     are row-major [out, in]; y = W x.
@@ -97,6 +106,9 @@ def tensor_specs(cfg: ModelConfig):
             specs.append((p + "bq", (1, cfg.n_q_heads * d), "normal"))
             specs.append((p + "bk", (1, cfg.n_kv_heads * d), "normal"))
             specs.append((p + "bv", (1, cfg.n_kv_heads * d), "normal"))
+        if cfg.qk_norm:
+            specs.append((p + "q_norm", (1, d), "gain"))
+            specs.append((p + "k_norm", (1, d), "gain"))
         specs.append((p + "wo", (H, cfg.n_q_heads * d), "normal"))
         specs.append((p + "ffn_norm", (1, H), "ones"))
         specs.append((p + "wg", (cfg.ffn_dim, H), "normal"))
@@ -108,18 +120,26 @@ def tensor_specs(cfg: ModelConfig):
     return specs
 
 
-def decode_bytes_per_token(cfg: ModelConfig, ctx: int) -> int:
+Q8_LAYER_MATRICES = ("wq", "wk", "wv", "wo", "wg", "wu", "wd")
+
+
+def decode_bytes_per_token(cfg: ModelConfig, ctx: int, q8: bool = False) -> int:
     """Algorithmic HBM bytes one decode step must read: every weight once plus
-    the K and V of `ctx` cached positions (bf16)."""
-    n = 0
+    the K and V of `ctx` cached positions (bf16).  With `q8` the per-layer
+    matrices whose input width is a whole number of 32-blocks are in the 8-bit
+    block format: 1 byte per code plus a 2-byte scale per 32 (17/16 bytes per
+    parameter); everything else stays bf16."""
+    n = 0.0
     for name, (r, c), _ in tensor_specs(cfg):
         if name == "embed":
-            n += cfg.hidden            # one embedding row is gathered
+            n += 2 * cfg.hidden            # one embedding row is gathered
+        elif q8 and name.split(".")[-1] in Q8_LAYER_MATRICES and c % 32 == 0:
+            n += r * c * 17 / 16
         else:
-            n += r * c
+            n += 2 * r * c
     if cfg.tied_embeddings:
-        n += cfg.vocab * cfg.hidden    # the LM head reads the (shared) embedding table
-    return 2 * n + cfg.n_layers * 2 * cfg.kv_dim * 2 * ctx
+        n += 2 * cfg.vocab * cfg.hidden    # the LM head reads the (shared) embedding table
+    return int(n) + cfg.n_layers * 2 * cfg.kv_dim * 2 * ctx
 
 
 def prefill_flops(cfg: ModelConfig, T: int, P: int = 0) -> float:

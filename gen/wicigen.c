@@ -65,6 +65,12 @@ void wicigen_normal_bf16(uint64_t seed, uint64_t tag, double std, uint64_t e0, u
     }
 }
 
+/* out[e] = bf16 bits of 1 + std * s_e (norm gains that are not all one), same stream rule. */
+void wicigen_gain_bf16(uint64_t seed, uint64_t tag, double std, uint64_t e0, uint64_t n, uint16_t *out) {
+    const uint64_t key = wicigen_stream(seed, tag);
+    for (uint64_t i = 0; i < n; ++i) out[i] = f32_to_bf16_rne((float)(1.0 + normal_at(key, e0 + i) * std));
+}
+
 /* out[e] = the same approximately-normal variates as doubles (for statistics tests). */
 void wicigen_normal_f64(uint64_t seed, uint64_t tag, uint64_t e0, uint64_t n, double *out) {
     const uint64_t key = wicigen_stream(seed, tag);

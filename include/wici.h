@@ -60,7 +60,22 @@ typedef struct wici_config {
     double rope_theta;
     int32_t tied_embeddings; /* 1: the LM head is the embedding table */
     int32_t qkv_bias;        /* 1: bq, bk, bv are present (added before RoPE) */
+    int32_t weight_format;   /* WICI_WEIGHTS_BF16, or WICI_WEIGHTS_Q8: the seven per-layer
+                                matrices in the 8-bit block format (see wici_load_weights_q8) */
+    int32_t qk_norm;         /* 1: Qwen3 block: each head of q and of k is RMS-normalised over
+                                head_dim with its own gain ("layers.<l>.q_norm" / ".k_norm",
+                                [1, head_dim]) before RoPE (the paper's models are Qwen3,
+                                Sec. 5.1, Tab. 1) */
+    int32_t max_sms;         /* SM share: the context's kernels use at most this many SMs
+                                (0: all).  Several contexts whose shares add up to at most
+                                the GPU's SM count decode concurrently, each on its own
+                                stream (Sec. 5.4, multiple clients; Sec. 7, task scheduling:
+                                the caller's stream priorities order the tenants). */
 } wici_config;
+
+/* Storage format of the per-layer matrices wq, wk, wv, wo, wg, wu, wd.  The
+ * embedding, norms, biases and LM head are bf16 in both. */
+enum { WICI_WEIGHTS_BF16 = 0, WICI_WEIGHTS_Q8 = 1 };
 
 /* Device bytes the caller allocates (each buffer 256-byte aligned). */
 typedef struct wici_sizes {
@@ -75,7 +90,7 @@ typedef struct wici_sizes {
  *   "layers.<l>.wk" / ".wv" [n_kv*d, hidden]; "layers.<l>.bq" [1, n_q*d] and
  *   ".bk" / ".bv" [1, n_kv*d] (qkv_bias only); "layers.<l>.wo" [hidden, n_q*d];
  *   "layers.<l>.ffn_norm" [1, hidden]; "layers.<l>.wg" / ".wu" [ffn, hidden];
- *   "layers.<l>.wd" [hidden, ffn].
+ *   "layers.<l>.wd" [hidden, ffn]; "layers.<l>.q_norm" / ".k_norm" [1, head_dim] (qk_norm only).
  * `data` is a host pointer (on_device = 0) or a device pointer (on_device = 1);
  * it is read during the call and not kept.  The paper's frameworks load a model
  * "tensor by tensor" (Sec. 4.1); so does this call. */
@@ -105,6 +120,33 @@ int wici_create(const wici_config *cfg, void *cuda_stream, void *weight_dev, voi
  * for RoPE, Wg/Wu rows are interleaved, Wq/Wk/Wv are concatenated).  May be
  * called several times; prefill/decode require every tensor to have been loaded. */
 int wici_load_weights(wici_ctx *ctx, const wici_tensor *t, int32_t n);
+
+/* One per-layer matrix in the 8-bit block format, GGUF-style (the paper's
+ * models are GGUF files at about 8.5 bits per parameter, Sec. 5.1 and Tab. 1):
+ * row r of a [rows, cols] matrix is cut into blocks of 32 consecutive input
+ * columns; block b holds 32 int8 codes (two's complement, in [-127, 127]) and
+ * one fp16 scale d[r][b], and stands for W[r][c] = d[r][c / 32] * code[r][c].
+ *   codes   int8 [rows, cols], row-major;   scales  fp16 bits [rows, cols / 32]
+ * Names and shapes are those of wici_tensor's per-layer matrices ("layers.<l>.wq",
+ * ".wk", ".wv", ".wo", ".wg", ".wu", ".wd").  `codes` and `scales` are host
+ * (on_device = 0) or device (on_device = 1) pointers, read during the call. */
+typedef struct wici_q8_tensor {
+    const char *name;
+    const void *codes;
+    const void *scales;
+    int64_t rows, cols;
+    int32_t on_device;
+} wici_q8_tensor;
+
+/* Copy `n` matrices in the 8-bit block format into the weight arena of a
+ * context created with weight_format = WICI_WEIGHTS_Q8 (the row pairings of
+ * wici_load_weights apply; each row's codes and scales are stored side by
+ * side).  Such a context takes the seven per-layer matrices only through this
+ * call, and the other tensors through wici_load_weights.  WICI_E_ARG for a
+ * bf16 context, an unknown name or a wrong shape; nothing is copied then.
+ * Constraints of the format here: hidden, ffn_dim and n_q_heads*head_dim
+ * multiples of 256. */
+int wici_load_weights_q8(wici_ctx *ctx, const wici_q8_tensor *t, int32_t n);
 
 /* Append `n` >= 1 host tokens at positions kv_len..kv_len+n-1 (Sec. 5.1 TTFT
  * path; a later call after decode steps is a chunked prefill onto the live cache).

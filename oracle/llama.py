@@ -25,6 +25,9 @@ and listed with the same wording in the design notes:
     activations that feed a prefill matrix product (h, q, o, h2, m) to bf16,
     a diagnostic that isolates operand rounding from errors.
   * QKV bias (Qwen2.5 shape) is added before RoPE; no other biases.
+  * Qwen3 block (`qk_norm`): each head of q and of k is RMS-normalised over
+    head_dim with its own gain (q_norm, k_norm), after the projection and
+    before RoPE.
   * Greedy token = argmax of the logits, lowest index on an exact tie.
   * Optional `q8_weights`: matrices in the 8-bit block format (oracle/q8.py)
     replace the bf16 tensors of the same name.
@@ -200,8 +203,13 @@ class OracleModel:
                 q = q + self._vec(p + "bq")
                 k = k + self._vec(p + "bk")
                 v = v + self._vec(p + "bv")
-            q = apply_rope(q.reshape(T, n_q, d), cos, sin)
-            k = apply_rope(k.reshape(T, n_kv, d), cos, sin)
+            q, k = q.reshape(T, n_q, d), k.reshape(T, n_kv, d)
+            if getattr(cfg, "qk_norm", False):
+                # Qwen3 block: every head of q and of k RMS-normalised over head_dim
+                q = rmsnorm(q, self._vec(p + "q_norm"), cfg.rms_eps)
+                k = rmsnorm(k, self._vec(p + "k_norm"), cfg.rms_eps)
+            q = apply_rope(q, cos, sin)
+            k = apply_rope(k, cos, sin)
             v = v.reshape(T, n_kv, d)
             self.K[l][:, P:P + T, :] = round_bf16(k).transpose(1, 0, 2)
             self.V[l][:, P:P + T, :] = round_bf16(v).transpose(1, 0, 2)

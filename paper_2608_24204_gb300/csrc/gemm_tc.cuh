@@ -15,6 +15,12 @@
 // warps fold each finished group into fp32 registers (round-to-nearest adds)
 // while the next group accumulates into the other buffer.
 //
+// Weights in the 8-bit block format arrive dequantised as WT = 3 bf16 terms
+// W = W_0 + W_1 + W_2 (exact: a code times an fp16 scale has at most 18
+// significant bits).  The K loop then runs once per weight term j, issuing the
+// products A_i W_j with i + j <= 2 (the others lie below 2^-24 of the result):
+// 3 + 2 + 1 MMAs per k-step instead of 3.
+//
 // Persistent: one CTA per SM walks the output tiles (M tiles fastest, so the
 // CTAs that run together share a weight tile through L2) with three warp roles:
 //   warp 0      TMA producer: 2-D tiled loads (128-byte swizzle) of the three A
@@ -121,11 +127,13 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, float *v) {
 
 // Epi::pair(t, c, v0, v1): output row t, columns (c, c + 1); Epi::row (when
 // Epi::kRow): the thread's whole span of columns at once, with vector stores
-template <int BN, class Epi>
+template <int BN, int WT, class Epi>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap map_a0, const __grid_constant__ CUtensorMap map_a1,
-                   const __grid_constant__ CUtensorMap map_a2, const __grid_constant__ CUtensorMap map_w, int T,
+                   const __grid_constant__ CUtensorMap map_a2, const __grid_constant__ CUtensorMap map_w,
+                   const __grid_constant__ CUtensorMap map_w1, const __grid_constant__ CUtensorMap map_w2, int T,
                    int N, int K, int *err, const Epi epi) {
+    static_assert(WT == 1 || WT == kTerms, "one exact bf16 weight term, or three");
     using G = TcTile<BN>;
     constexpr int S = G::STAGES;
     extern __shared__ uint8_t smem_raw[];
@@ -137,7 +145,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     const int ntm = (T + TC_BM - 1) / TC_BM, ntn = (N + BN - 1) / BN;
     const int ntiles = ntm * ntn;
     const int nk = (K + TC_BK - 1) / TC_BK;
-    const int ngroups = (nk + TC_GROUP - 1) / TC_GROUP;
+    const int nkk = nk * WT;                      // k-blocks of all weight terms
+    const int ngroups = (nkk + TC_GROUP - 1) / TC_GROUP;
     const uint32_t base = (smem_u32(smem_raw) + 1023u) & ~1023u;
 
     if (threadIdx.x == 0) {
@@ -169,17 +178,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             bool ok = true;
             for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
                 const int m0 = (tile % ntm) * TC_BM, n0 = (tile / ntm) * BN;
-                for (int kb = 0; kb < nk; ++kb, ++it) {
+                for (int kk = 0; kk < nkk; ++kk, ++it) {
                     const int s = it % S;
                     if (it >= S && !(ok = mbar_wait(smem_u32(&empty_bar[s]), ((it / S) + 1) & 1, err, SITE_TC_EMPTY)))
                         break;
+                    const int j = WT == 1 ? 0 : kk / nk, kb = kk - j * nk;     // weight term, k-block
                     const uint32_t st = base + (uint32_t)s * G::STAGE_BYTES;
                     const uint32_t fb = smem_u32(&full_bar[s]);
-                    mbar_arrive_expect_tx(fb, G::STAGE_BYTES);
+                    // term j meets the activation terms i <= 2 - j only
+                    mbar_arrive_expect_tx(fb, (uint32_t)(kTerms - j) * TC_A_BYTES + G::B_BYTES);
                     tma_load_2d(st, &map_a0, kb * TC_BK, m0, fb);
-                    tma_load_2d(st + TC_A_BYTES, &map_a1, kb * TC_BK, m0, fb);
-                    tma_load_2d(st + 2 * TC_A_BYTES, &map_a2, kb * TC_BK, m0, fb);
-                    tma_load_2d(st + kTerms * TC_A_BYTES, &map_w, kb * TC_BK, n0, fb);
+                    if (j < 2) tma_load_2d(st + TC_A_BYTES, &map_a1, kb * TC_BK, m0, fb);
+                    if (j < 1) tma_load_2d(st + 2 * TC_A_BYTES, &map_a2, kb * TC_BK, m0, fb);
+                    tma_load_2d(st + kTerms * TC_A_BYTES, j == 0 ? &map_w : j == 1 ? &map_w1 : &map_w2, kb * TC_BK, n0,
+                                fb);
                     s_issued = it + 1;
                 }
             }
@@ -197,12 +209,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         break;
                     tc_fence_after();
                     const uint32_t acc = tmem + (uint32_t)(b * BN);
-                    const int kb1 = min(nk, (gi + 1) * TC_GROUP);
-                    for (int kb = gi * TC_GROUP; kb < kb1; ++kb, ++it) {
+                    const int kk1 = min(nkk, (gi + 1) * TC_GROUP);
+                    for (int kk = gi * TC_GROUP; kk < kk1; ++kk, ++it) {
                         const int s = it % S;
                         ok = mbar_wait(smem_u32(&full_bar[s]), (it / S) & 1, err, SITE_TC_FULL);
                         if (!ok) break;
                         tc_fence_after();
+                        const int nt = WT == 1 ? kTerms : kTerms - kk / nk;   // activation terms meeting this weight term
                         const uint32_t st = base + (uint32_t)s * G::STAGE_BYTES;
                         // descriptors of k-step 0; each k-step of 16 elements is 32 bytes further
                         const uint64_t bd0 = tc_desc_sw128(st + kTerms * TC_A_BYTES);
@@ -211,8 +224,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         for (int k = 0; k < TC_BK / 16; ++k)
 #pragma unroll
                             for (int t = 0; t < kTerms; ++t)
-                                tc_mma(acc, ad0 + (uint64_t)((t * TC_A_BYTES + 32 * k) >> 4), bd0 + (uint64_t)(2 * k),
-                                       idesc, (kb != gi * TC_GROUP || k != 0 || t != 0));
+                                if (t < nt)
+                                    tc_mma(acc, ad0 + (uint64_t)((t * TC_A_BYTES + 32 * k) >> 4),
+                                           bd0 + (uint64_t)(2 * k), idesc, (kk != gi * TC_GROUP || k != 0 || t != 0));
                         tc_commit(smem_u32(&empty_bar[s]));
                     }
                     tc_commit(smem_u32(&acc_full[b]));  // fires when this group's MMAs have completed

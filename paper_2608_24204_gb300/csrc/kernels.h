@@ -35,6 +35,12 @@ struct Bufs {
     uint16_t *A[kTerms];  // RMSNorm output                                   [max_chunk][H]
     uint16_t *O[kTerms];  // attention output                                 [max_chunk][qdim]
     uint16_t *M[kTerms];  // SwiGLU output                                    [max_chunk][F]
+    // 8-bit block format only: the matrix of the next prefill GEMM dequantised
+    // as three bf16 terms (exact: a code times an fp16 scale has <= 18 significant bits)
+    uint16_t *Wt[kTerms]; //                                                    [wt_elems]
+    // qk_norm only: k of this decode step before its norm and RoPE            [kvdim]
+    // and the prefill chunk's q | k before their norms and RoPE               [max_chunk][qdim + kvdim]
+    float *kraw, *QKraw;
 };
 
 // TMA descriptors of the prefill GEMM operands (built once per context).
@@ -43,8 +49,10 @@ struct PrefillMaps {
     CUtensorMap q[kTerms];                             // queries: [token][head][d], group x tpt boxes
     CUtensorMap kv;                                    // the whole KV pool: [page][K|V][kv_head][16][d]
     std::vector<CUtensorMap> wqkv, wo, wgu, wd;        // per layer weights, boxes of bn_* rows
+    CUtensorMap wt_qkv[kTerms], wt_o[kTerms], wt_gu[kTerms], wt_d[kTerms];  // 8-bit format: the dequantised terms
     int bn_qkv, bn_o, bn_gu, bn_d;                     // output-tile width of each matrix's GEMM
 };
+
 
 // Encodes every tensor map of `m`; returns an error message or nullptr.
 const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m);

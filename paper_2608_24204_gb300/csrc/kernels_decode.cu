@@ -8,9 +8,12 @@
 // warps do the dot products with the input vector held in registers.  The
 // producer starts before griddepcontrol.wait, so under programmatic dependent
 // launch a GEMV's first weight tiles stream in while its predecessor finishes.
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
+
+#include <type_traits>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -66,6 +69,7 @@ struct EpiQKV {
     const float2 *rope;
     const int *ctrl;
     const uint16_t *bias;  // packed like the rows, or nullptr
+    float *kraw;           // qk_norm: q and k leave unnormalised and without RoPE (k here)
     int qdim, kvdim, d, nkv;
     size_t page_elems;
     static constexpr bool kArgmax = false;
@@ -79,7 +83,13 @@ struct EpiQKV {
         const int pos = ctrl[CTRL_POS];
         uint16_t *page = kv + (size_t)pages[pos / kPage] * page_elems;
         const int slot = pos % kPage;
-        if (r0 < qdim + kvdim) {
+        if (kraw && r0 < qdim + kvdim) {
+            // the per-head norm needs the whole head: the attention phase finishes q and k
+            const int hd = r0 / d, i = (r0 % d) >> 1, half = d >> 1;
+            float *dst = r0 < qdim ? q + hd * d : kraw + (hd - qdim / d) * d;
+            dst[i] = a;
+            dst[i + half] = b;
+        } else if (r0 < qdim + kvdim) {
             const int hd = r0 / d, i = (r0 % d) >> 1, half = d >> 1;
             const float2 cs = rope[(size_t)pos * half + i];
             const float ra = a * cs.x - b * cs.y;
@@ -185,6 +195,40 @@ __device__ __forceinline__ float dot8(const uint4 w, const float *h, float a) {
     a = fmaf(bf16lo(w.w), h[6], a);
     a = fmaf(bf16hi(w.w), h[7], a);
     return a;
+}
+
+// ------------------------------------------------- 8-bit block rows (decode) --
+// A row of the 8-bit block format in shared memory: K int8 codes (two's
+// complement), then the row's K/32 fp16 block scales.
+//
+// The input vector of a phase is put once into 24-bit fixed point,
+// X[c] = rint(h[c] * 2^E) with |X| < 2^23 (E from the vector's largest
+// magnitude, one rounding of at most 2^-24 of it), and X is cut into three
+// byte digits X = 65536 X2 + 256 X1 + X0 (X2 signed, X1 and X0 unsigned).  The
+// integer dot products of 16 codes with each digit (dp4a, exact in int32) make
+// the chunk's exact sum q . X, which one fp32 rounding carries into the row's
+// fp32 accumulator with the block scale; 2^-E is applied once per row.  That is
+// 12 dp4a and a handful of fp32 operations per 16 codes, where converting every
+// code to fp32 costs three operations per code.
+__device__ __forceinline__ int dp4a_ss(uint32_t a, uint32_t b, int c) {
+    int d;
+    asm("dp4a.s32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+__device__ __forceinline__ int dp4a_su(uint32_t a, uint32_t b, int c) {
+    int d;
+    asm("dp4a.s32.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+    return d;
+}
+// exact int -> fp32 for |v| < 2^22: the integer added under the exponent of 1.5 * 2^23
+__device__ __forceinline__ float small_int_to_f32(int v) {
+    return __int_as_float(0x4B400000 + v) - 12582912.0f;
+}
+
+__device__ __forceinline__ float lds_f16(uint32_t addr) {
+    unsigned short v;
+    asm volatile("ld.shared.u16 %0, [%1];" : "=h"(v) : "r"(addr));
+    return __half2float(__ushort_as_half(v));
 }
 
 // ------------------------------------------------------------------- GEMV ----
@@ -753,6 +797,7 @@ struct GShape {
 
 struct MegaArgs {
     const uint16_t *W;          // weight arena
+    float *kraw;                // qk_norm: this step's k before its norm and RoPE [kvdim], else nullptr
     size_t lstride;             // elements between the same tensor of consecutive layers
     LayerOffsets l0;            // layer 0 offsets
     size_t w_embed, w_final_norm, w_lm;
@@ -785,37 +830,39 @@ __device__ __forceinline__ int mega_unit(uint32_t b, int n_units) {
 }
 
 // ----------------------------------------------------------- producer side --
-__device__ bool mp_rows(MegaRing &R, const uint16_t *W, int K, int n_units, int rpu, int RPS, int *err,
-                        uint64_t pol) {
+// this CTA's rows of an n_units-unit matrix whose rows are row_bytes long (bf16:
+// 2K; the 8-bit block format: q8_row_bytes(K)), RPS rows per ring slot
+__device__ bool mp_rows(MegaRing &R, const uint16_t *W, uint32_t row_bytes, int n_units, int rpu, int RPS,
+                        int *err, uint64_t pol) {
     const int u0 = mega_unit(R.b0, n_units);
     const int u1 = mega_unit(R.b1, n_units);
     const int total_rows = (u1 - u0) * rpu;
     const int nst = (total_rows + RPS - 1) / RPS;
-    const uint16_t *src = W + (size_t)u0 * rpu * K;
+    const uint8_t *src = reinterpret_cast<const uint8_t *>(W) + (size_t)u0 * rpu * row_bytes;
     for (int s = 0; s < nst; ++s) {
         const int slot = R.n % kMegaSlots;
         if (R.n >= kMegaSlots &&
             !mbar_wait(R.empty0 + 8 * slot, ((R.n / kMegaSlots) + 1) & 1, err, SITE_MEGA_EMPTY))
             return false;
         const int rows = min(RPS, total_rows - s * RPS);
-        const uint32_t bytes = (uint32_t)rows * (uint32_t)K * 2u;
+        const uint32_t bytes = (uint32_t)rows * row_bytes;
         mbar_arrive_expect_tx(R.full0 + 8 * slot, bytes);
-        bulk_g2s(R.data0 + slot * kMegaSlotBytes, src + (size_t)s * RPS * K, bytes, R.full0 + 8 * slot, pol);
+        bulk_g2s(R.data0 + slot * kMegaSlotBytes, src + (size_t)s * RPS * row_bytes, bytes, R.full0 + 8 * slot, pol);
         ++R.n;
     }
     return true;
 }
 
 // move rows [skip, skip + bytes) of this CTA's share of a GEMV phase into L2
-__device__ void mp_prefetch(const MegaRing &R, const uint16_t *W, int K, int n_units, int rpu, size_t skip,
-                            size_t bytes) {
+__device__ void mp_prefetch(const MegaRing &R, const uint16_t *W, uint32_t row_bytes, int n_units, int rpu,
+                            size_t skip, size_t bytes) {
     const int u0 = mega_unit(R.b0, n_units);
     const int u1 = mega_unit(R.b1, n_units);
-    const size_t row = (size_t)K * 2;
+    const size_t row = row_bytes;
     const size_t own = (size_t)(u1 - u0) * rpu * row;
     skip -= skip % row;
     const size_t end = own < skip + bytes ? own : skip + bytes;
-    const uint8_t *src = reinterpret_cast<const uint8_t *>(W + (size_t)u0 * rpu * K);
+    const uint8_t *src = reinterpret_cast<const uint8_t *>(W) + (size_t)u0 * rpu * row;
     for (size_t off = skip; off < end; off += 32768)
         bulk_prefetch_l2(src + off, (uint32_t)(end - off < 32768 ? end - off : 32768));
 }
@@ -1029,14 +1076,230 @@ __device__ bool mc_gemv(MegaRing &R, float *red, int K, int n_units, int rpu, co
     return true;
 }
 
+// One GEMV phase over a matrix in the 8-bit block format (rows of
+// q8_row_bytes(K) bytes), same role as mc_gemv.  Thread t owns the 16-element
+// chunks c = t + 256 j of the input, as byte digits of its fixed-point form.
+template <class QS, class Epi>
+__device__ bool mc_gemv_q8(MegaRing &R, float *red, int K, int n_units, int rpu, const float *in,
+                           const uint16_t *gain, const uint16_t *embed, float *x_out, float eps, int *ctrl, Epi &epi,
+                           float *s_part) {
+    constexpr int NCH = QS::NCH, RPS = QS::RPS;
+    constexpr bool FULL = QS::FULL;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int u0 = mega_unit(R.b0, n_units);
+    const int u1 = mega_unit(R.b1, n_units);
+    const int total_rows = (u1 - u0) * rpu;
+    const int nst = (total_rows + RPS - 1) / RPS;
+    int *err = ctrl + CTRL_ERR;
+    const int nchunks = K >> 4;
+    float h[NCH][16];
+    float ss = 0.f;
+    const int tok = embed ? ctrl[CTRL_TOKEN] : 0;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+        const int c = tid + kGemvConsumers * j;
+        if (FULL || c < nchunks) {
+            if (embed) {
+#pragma unroll
+                for (int hv = 0; hv < 2; ++hv) {
+                    const uint4 w = *reinterpret_cast<const uint4 *>(embed + (size_t)tok * K + c * 16 + hv * 8);
+                    float *d = h[j] + hv * 8;
+                    d[0] = bf16lo(w.x); d[1] = bf16hi(w.x); d[2] = bf16lo(w.y); d[3] = bf16hi(w.y);
+                    d[4] = bf16lo(w.z); d[5] = bf16hi(w.z); d[6] = bf16lo(w.w); d[7] = bf16hi(w.w);
+                }
+                if (blockIdx.x == 0) {
+                    float4 *dst = reinterpret_cast<float4 *>(x_out + c * 16);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        dst[q] = make_float4(h[j][4 * q], h[j][4 * q + 1], h[j][4 * q + 2], h[j][4 * q + 3]);
+                }
+            } else {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float4 a = __ldcg(reinterpret_cast<const float4 *>(in + c * 16 + 4 * q));
+                    h[j][4 * q] = a.x; h[j][4 * q + 1] = a.y; h[j][4 * q + 2] = a.z; h[j][4 * q + 3] = a.w;
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < 16; ++e) ss = fmaf(h[j][e], h[j][e], ss);
+        } else {
+#pragma unroll
+            for (int e = 0; e < 16; ++e) h[j][e] = 0.f;
+        }
+    }
+    if (gain) {
+        ss = warp_sum(ss);
+        if (lane == 0) s_part[warp] = ss;
+        consumer_sync();
+        float tot = 0.f;
+#pragma unroll
+        for (int w = 0; w < kGemvWarps; ++w) tot += s_part[w];
+        const float rinv = 1.0f / sqrtf(tot / (float)K + eps);
+#pragma unroll
+        for (int j = 0; j < NCH; ++j) {
+            const int c = tid + kGemvConsumers * j;
+            if (FULL || c < nchunks) {
+#pragma unroll
+                for (int hv = 0; hv < 2; ++hv) {
+                    const uint4 gw = *reinterpret_cast<const uint4 *>(gain + c * 16 + hv * 8);
+                    const float gg[8] = {bf16lo(gw.x), bf16hi(gw.x), bf16lo(gw.y), bf16hi(gw.y),
+                                         bf16lo(gw.z), bf16hi(gw.z), bf16lo(gw.w), bf16hi(gw.w)};
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) h[j][hv * 8 + e] = h[j][hv * 8 + e] * rinv * gg[e];
+                }
+            }
+        }
+    }
+    // fixed point: M * 2^E in [2^22, 2^23) for the largest magnitude M
+    float mx = 0.f;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j)
+#pragma unroll
+        for (int e = 0; e < 16; ++e) mx = fmaxf(mx, fabsf(h[j][e]));
+    mx = warp_max(mx);
+    consumer_sync();   // the RMSNorm reads of s_part are done
+    if (lane == 0) s_part[warp] = mx;
+    consumer_sync();
+    float M = 0.f;
+#pragma unroll
+    for (int w = 0; w < kGemvWarps; ++w) M = fmaxf(M, s_part[w]);
+    const int E = M > 0.f ? min(22 - ilogbf(M), 120) : 0;
+    const float to_fixed = ldexpf(1.0f, E), from_fixed = ldexpf(1.0f, -E);
+    uint32_t dg[NCH][3][4];   // [chunk][digit X2, X1, X0][4 words of 4 byte digits]
+#pragma unroll
+    for (int j = 0; j < NCH; ++j)
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            uint32_t w2 = 0, w1 = 0, w0 = 0;
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                const int X = max(min(__float2int_rn(h[j][4 * k + b] * to_fixed), (1 << 23) - 1), -(1 << 23) + 1);
+                w2 |= ((uint32_t)(X >> 16) & 0xFFu) << (8 * b);
+                w1 |= ((uint32_t)(X >> 8) & 0xFFu) << (8 * b);
+                w0 |= ((uint32_t)X & 0xFFu) << (8 * b);
+            }
+            dg[j][0][k] = w2;
+            dg[j][1][k] = w1;
+            dg[j][2][k] = w0;
+        }
+
+    const uint32_t row_bytes = (uint32_t)q8_row_bytes((size_t)K);
+    const bool tail_ok = FULL || tid + kGemvConsumers * (NCH - 1) < nchunks;
+    int buf = 0, brow = 0, bunit0 = 0;
+    bool ok = true;
+    for (int s = 0; s < nst; ++s) {
+        const int slot = R.n % kMegaSlots;
+        const int rows = min(RPS, total_rows - s * RPS);
+        ok = ok && !*reinterpret_cast<volatile int *>(R.abort) &&
+             mbar_wait(R.full0 + 8 * slot, (R.n / kMegaSlots) & 1, err, SITE_MEGA_FULL);
+        if (!ok) *R.abort = 1;
+        float acc[RPS];
+#pragma unroll
+        for (int r = 0; r < RPS; ++r) acc[r] = 0.f;
+        // chunk c: codes at byte 16 c of the row, its block's scale at byte K + 2 (c / 2)
+        const uint32_t s0 = R.data0 + (uint32_t)slot * kMegaSlotBytes;
+        const uint32_t sb = s0 + (uint32_t)tid * 16u;
+        const uint32_t sc = s0 + (uint32_t)K + (uint32_t)(tid >> 1) * 2u;
+        if (ok) {
+#pragma unroll
+            for (int r = 0; r < RPS; ++r)
+                if (rows == RPS || r < rows)
+#pragma unroll
+                    for (int j = 0; j < NCH; ++j)
+                        if (j < NCH - 1 || tail_ok) {
+                            const uint4 w = lds128(sb + r * row_bytes + j * kGemvConsumers * 16);
+                            const float d = lds_f16(sc + r * row_bytes + j * (kGemvConsumers / 2) * 2);
+                            int a2 = dp4a_ss(w.x, dg[j][0][0], 0), a1 = dp4a_su(w.x, dg[j][1][0], 0),
+                                a0 = dp4a_su(w.x, dg[j][2][0], 0);
+                            a2 = dp4a_ss(w.y, dg[j][0][1], a2); a1 = dp4a_su(w.y, dg[j][1][1], a1);
+                            a0 = dp4a_su(w.y, dg[j][2][1], a0);
+                            a2 = dp4a_ss(w.z, dg[j][0][2], a2); a1 = dp4a_su(w.z, dg[j][1][2], a1);
+                            a0 = dp4a_su(w.z, dg[j][2][2], a0);
+                            a2 = dp4a_ss(w.w, dg[j][0][3], a2); a1 = dp4a_su(w.w, dg[j][1][3], a1);
+                            a0 = dp4a_su(w.w, dg[j][2][3], a0);
+                            const float cv = fmaf(small_int_to_f32(a2), 65536.0f,
+                                                  fmaf(small_int_to_f32(a1), 256.0f, small_int_to_f32(a0)));
+                            acc[r] = fmaf(d, cv, acc[r]);
+                        }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(R.empty0 + 8 * slot);
+        ++R.n;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+            for (int r = 0; r < RPS; ++r) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
+        if (lane == 0) {
+            float *rb = red + (size_t)(buf * kGemvWarps + warp) * kRedRows + brow;
+#pragma unroll
+            for (int r = 0; r < RPS; ++r)
+                if (r < rows) rb[r] = acc[r];
+        }
+        brow += rows;
+        if (s == nst - 1 || brow + RPS > kRedRows) {
+            if (consumer_sync_or(!ok)) return false;
+            const int bunits = brow / rpu;
+            for (int t = tid; t < bunits; t += kGemvConsumers) {
+                float v[2];
+                for (int j = 0; j < rpu; ++j) {
+                    float sum = 0.f;
+#pragma unroll
+                    for (int w = 0; w < kGemvWarps; ++w)
+                        sum += red[(size_t)(buf * kGemvWarps + w) * kRedRows + t * rpu + j];
+                    v[j] = sum * from_fixed;
+                }
+                epi.unit(u0 + bunit0 + t, v);
+            }
+            bunit0 += bunits;
+            brow = 0;
+            buf ^= 1;
+        }
+    }
+    return true;
+}
+
+// a per-layer GEMV phase in the layer matrices' format
+template <bool Q8, class S, class Epi>
+__device__ __forceinline__ bool mc_layer_gemv(MegaRing &R, float *red, int K, int n_units, int rpu, const float *in,
+                                              const uint16_t *gain, const uint16_t *embed, float *x_out, float eps,
+                                              int *ctrl, Epi &epi, float *s_part) {
+    if constexpr (Q8)
+        return mc_gemv_q8<S>(R, red, K, n_units, rpu, in, gain, embed, x_out, eps, ctrl, epi, s_part);
+    else
+        return mc_gemv<S>(R, red, K, n_units, rpu, in, gain, embed, x_out, eps, ctrl, epi, s_part);
+}
+
 // Attention of the current token for this CTA's split (KV head g, pages
 // [p0, p0 + n)), then the split state to global memory and the ticket; the last
 // split of head g combines the states in split order into o.  Warp (j, set) with
 // j = warp % group handles query head g*group + j on pages i = set (mod wph);
 // warps beyond group * wph only keep the ring in step.
+// Qwen3 block, for one head held by a warp (lane l has elements l*EPL ..): RMS
+// norm over the head with the gain, then rotate-half RoPE at position pos (the
+// partner of element i < D/2 is i + D/2, EPL elements further in lane l + 16).
+template <int D>
+__device__ __forceinline__ void head_norm_rope(float *v, const uint16_t *gain, float eps, const float2 *rope,
+                                               int pos, int lane) {
+    constexpr int EPL = D / 32, HALF = D / 2;
+    float ss = 0.f;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) ss = fmaf(v[e], v[e], ss);
+    const float rinv = 1.0f / sqrtf(warp_sum(ss) / (float)D + eps);
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) v[e] = v[e] * rinv * bf16_to_f32(gain[lane * EPL + e]);
+    const bool lower = lane < 16;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) {
+        const float other = __shfl_xor_sync(0xffffffffu, v[e], 16);
+        const int i = (lane * EPL + e) % HALF;
+        const float2 cs = rope[(size_t)pos * HALF + i];
+        v[e] = lower ? v[e] * cs.x - other * cs.y : v[e] * cs.x + other * cs.y;
+    }
+}
+
 template <int D>
 __device__ bool mc_attn(MegaRing &R, const MegaArgs &a, const uint16_t *kvl, const MegaSplit &sp, int len,
-                        float (*s_state)[D + 4], int *s_last) {
+                        float (*s_state)[D + 4], int *s_last, const uint16_t *qn, const uint16_t *kn) {
     constexpr int EPL = D / 32;
     constexpr uint32_t BLK = kPage * D * 2;
     constexpr int STRIDE = D + 4;
@@ -1053,21 +1316,44 @@ __device__ bool mc_attn(MegaRing &R, const MegaArgs &a, const uint16_t *kvl, con
     if (qwarp) {
         if constexpr (EPL == 4) {
             const float4 q4 = __ldcg(reinterpret_cast<const float4 *>(a.q + head * D + lane * 4));
-            qv[0] = q4.x * a.qscale; qv[1] = q4.y * a.qscale; qv[2] = q4.z * a.qscale; qv[3] = q4.w * a.qscale;
+            qv[0] = q4.x; qv[1] = q4.y; qv[2] = q4.z; qv[3] = q4.w;
         } else {
             const float2 q2 = __ldcg(reinterpret_cast<const float2 *>(a.q + head * D + lane * 2));
-            qv[0] = q2.x * a.qscale; qv[1] = q2.y * a.qscale;
+            qv[0] = q2.x; qv[1] = q2.y;
         }
+        if (qn) head_norm_rope<D>(qv, qn, a.eps, a.rope, len - 1, lane);
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) qv[e] *= a.qscale;
     }
     // this step's K/V row was written by another CTA during the QKV phase, possibly
     // after the producer copied its page: it is read from L2 instead of the ring
+    // (with qk_norm the key is finished here from its raw form and written to the page)
     const int cur_slot = (len - 1) % kPage;
     uint32_t kcur[EPL / 2], vcur[EPL / 2];
     if (qwarp && sp.p0 + sp.n == sp.npages) {
         const int page = a.pages[sp.npages - 1];
-        const uint16_t *kr = kvl + (size_t)page * a.page_elems + ((size_t)sp.g * kPage + cur_slot) * D + lane * EPL;
+        uint16_t *kr = const_cast<uint16_t *>(kvl) + (size_t)page * a.page_elems + ((size_t)sp.g * kPage + cur_slot) * D +
+                       lane * EPL;
         const uint16_t *vr = kr + (size_t)a.nkv * kPage * D;
-        if constexpr (EPL == 4) {
+        if (kn) {
+            float kv_[EPL];
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) kv_[e] = __ldcg(a.kraw + sp.g * D + lane * EPL + e);
+            head_norm_rope<D>(kv_, kn, a.eps, a.rope, len - 1, lane);
+#pragma unroll
+            for (int e = 0; e < EPL; e += 2)
+                kcur[e >> 1] = (uint32_t)f32_to_bf16(kv_[e]) | ((uint32_t)f32_to_bf16(kv_[e + 1]) << 16);
+            if (w == 0) {
+#pragma unroll
+                for (int e = 0; e < EPL; e += 2) reinterpret_cast<uint32_t *>(kr)[e >> 1] = kcur[e >> 1];
+            }
+            if constexpr (EPL == 4) {
+                const uint2 v2 = __ldcg(reinterpret_cast<const uint2 *>(vr));
+                vcur[0] = v2.x; vcur[1] = v2.y;
+            } else {
+                vcur[0] = __ldcg(reinterpret_cast<const unsigned int *>(vr));
+            }
+        } else if constexpr (EPL == 4) {
             const uint2 k2 = __ldcg(reinterpret_cast<const uint2 *>(kr));
             const uint2 v2 = __ldcg(reinterpret_cast<const uint2 *>(vr));
             kcur[0] = k2.x; kcur[1] = k2.y; vcur[0] = v2.x; vcur[1] = v2.y;
@@ -1272,8 +1558,17 @@ __device__ void mega_rebalance(const MegaArgs &a, float *rate) {
     }
 }
 
-template <int D, class SH, class SF>
+// SH, SF: GEMV shapes of K = hidden and K = ffn for bf16 rows; with Q8 the seven
+// per-layer matrices are in the 8-bit block format and stream with the shapes
+// QH, QF (16-element chunks, rows per slot sized for the shorter rows), while
+// the LM head stays bf16 (SH).
+template <int D, class SH, class SF, bool Q8, class QH, class QF>
 __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const MegaArgs a) {
+    using LH = std::conditional_t<Q8, QH, SH>;   // layer matrices with K = hidden (and K = n_q * d)
+    using LF = std::conditional_t<Q8, QF, SF>;   // the down projection, K = ffn
+    const uint32_t rb_h = Q8 ? (uint32_t)q8_row_bytes((size_t)a.H) : (uint32_t)a.H * 2u;
+    const uint32_t rb_q = Q8 ? (uint32_t)q8_row_bytes((size_t)a.qdim) : (uint32_t)a.qdim * 2u;
+    const uint32_t rb_f = Q8 ? (uint32_t)q8_row_bytes((size_t)a.F) : (uint32_t)a.F * 2u;
     extern __shared__ __align__(128) uint8_t smem[];
     float *red = reinterpret_cast<float *>(smem);
     __shared__ __align__(8) uint64_t bars[2 * kMegaSlots];
@@ -1316,13 +1611,13 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
             bool ok = true;
             for (int l = 0; l < a.L && ok; ++l) {
                 const size_t lo = (size_t)l * a.lstride;
-                ok = mp_rows(R, a.W + a.l0.wqkv + lo, a.H, a.nqkv / 2, 2, SH::RPS, err, pol) &&
+                ok = mp_rows(R, a.W + a.l0.wqkv + lo, rb_h, a.nqkv / 2, 2, LH::RPS, err, pol) &&
                      mp_pages<D>(R, a, a.KV + (size_t)l * a.kv_layer_elems, sp, err) &&
-                     mp_rows(R, a.W + a.l0.wo + lo, a.qdim, a.H, 1, SH::RPS, err, pol) &&
-                     mp_rows(R, a.W + a.l0.wgu + lo, a.H, a.F, 2, SH::RPS, err, pol) &&
-                     mp_rows(R, a.W + a.l0.wd + lo, a.F, a.H, 1, SF::RPS, err, pol);
+                     mp_rows(R, a.W + a.l0.wo + lo, rb_q, a.H, 1, LH::RPS, err, pol) &&
+                     mp_rows(R, a.W + a.l0.wgu + lo, rb_h, a.F, 2, LH::RPS, err, pol) &&
+                     mp_rows(R, a.W + a.l0.wd + lo, rb_f, a.H, 1, LF::RPS, err, pol);
             }
-            if (ok) mp_rows(R, a.W + a.w_lm, a.H, a.V, 1, SH::RPS, err, pol);
+            if (ok) mp_rows(R, a.W + a.w_lm, (uint32_t)a.H * 2u, a.V, 1, SH::RPS, err, pol);
             // no copy may still be landing in shared memory when the CTA exits
             for (int s = max(0, R.n - kMegaSlots); s < R.n; ++s)
                 mbar_wait(R.full0 + 8 * (s % kMegaSlots), (s / kMegaSlots) & 1, err, SITE_MEGA_DRAIN);
@@ -1342,29 +1637,32 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
         EpiQKV eq;
         eq.q = a.q; eq.kv = kvl; eq.pages = a.pages; eq.rope = a.rope; eq.ctrl = a.ctrl;
         eq.bias = a.bias ? a.W + a.l0.bqkv + lo : nullptr;
+        eq.kraw = a.kraw;
         eq.qdim = a.qdim; eq.kvdim = a.kvdim; eq.d = a.d; eq.nkv = a.nkv; eq.page_elems = a.page_elems;
-        ok = mc_gemv<SH>(R, red, a.H, a.nqkv / 2, 2, a.x, a.W + a.l0.attn_norm + lo,
-                         l == 0 ? a.W + a.w_embed : nullptr, a.x, a.eps, a.ctrl, eq, s_part) &&
+        ok = mc_layer_gemv<Q8, LH>(R, red, a.H, a.nqkv / 2, 2, a.x, a.W + a.l0.attn_norm + lo,
+                                   l == 0 ? a.W + a.w_embed : nullptr, a.x, a.eps, a.ctrl, eq, s_part) &&
              mega_grid_sync(a.ctrl, ++k, &s_flag);
         if (!ok) break;
         // the attention phase leaves the HBM nearly idle: move the first gate/up rows
         // of this CTA into L2 meanwhile (its O rows are already filling the ring)
-        if (tid == 0) mp_prefetch(R, a.W + a.l0.wgu + lo, a.H, a.F, 2, 0, kMegaPrefetchBytes);
-        ok = mc_attn<D>(R, a, kvl, sp, len, s_state, &s_last) &&
+        if (tid == 0) mp_prefetch(R, a.W + a.l0.wgu + lo, rb_h, a.F, 2, 0, kMegaPrefetchBytes);
+        ok = mc_attn<D>(R, a, kvl, sp, len, s_state, &s_last, a.kraw ? a.W + a.l0.qn + lo : nullptr,
+                        a.kraw ? a.W + a.l0.kn + lo : nullptr) &&
              mega_grid_sync(a.ctrl, ++k, &s_flag);
         if (!ok) break;
         EpiResidual er{a.x};
-        ok = mc_gemv<SH>(R, red, a.qdim, a.H, 1, a.o, nullptr, nullptr, nullptr, a.eps, a.ctrl, er, s_part) &&
+        ok = mc_layer_gemv<Q8, LH>(R, red, a.qdim, a.H, 1, a.o, nullptr, nullptr, nullptr, a.eps, a.ctrl, er,
+                                   s_part) &&
              mega_grid_sync(a.ctrl, ++k, &s_flag);
         if (!ok) break;
         EpiSwiGLU es{a.m};
         const uint64_t t_gu = globaltimer_ns();
-        ok = mc_gemv<SH>(R, red, a.H, a.F, 2, a.x, a.W + a.l0.ffn_norm + lo, nullptr, nullptr, a.eps, a.ctrl, es,
-                         s_part);
+        ok = mc_layer_gemv<Q8, LH>(R, red, a.H, a.F, 2, a.x, a.W + a.l0.ffn_norm + lo, nullptr, nullptr, a.eps,
+                                   a.ctrl, es, s_part);
         gu_ns += globaltimer_ns() - t_gu;
         ok = ok && mega_grid_sync(a.ctrl, ++k, &s_flag);
         if (!ok) break;
-        ok = mc_gemv<SF>(R, red, a.F, a.H, 1, a.m, nullptr, nullptr, nullptr, a.eps, a.ctrl, er, s_part);
+        ok = mc_layer_gemv<Q8, LF>(R, red, a.F, a.H, 1, a.m, nullptr, nullptr, nullptr, a.eps, a.ctrl, er, s_part);
     }
     if (tid == 0) a.cta_time[blockIdx.x] = (float)gu_ns * 1e-3f;
     if (ok) ok = mega_grid_sync(a.ctrl, ++k, &s_flag);
@@ -1406,6 +1704,10 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
             a.ctrl[CTRL_POS] = np;
             a.hist[np] = fi;
             a.ctrl[CTRL_LM_TICKET] = 0;
+            // every CTA has passed the last grid barrier (it took a ticket after it):
+            // the arrival counter starts the next step at zero without a memset in the
+            // stream (a memset would queue behind other streams' copies and kernels)
+            a.ctrl[CTRL_GRID_BAR] = 0;
         }
         s_last = (t == (int)gridDim.x - 1);
     }
@@ -1501,17 +1803,30 @@ using MegaF8192 = GShape<4, 2, true>;
 using MegaH5120 = GShape<3, 2, false>;    // Qwen2.5-14B widths: hidden 5120, ffn 13824
 using MegaF13824 = GShape<7, 1, false>;
 using MegaSmall = GShape<1, 8, false>;    // hidden and ffn below 2048 (e.g. 256 / 688)
-#define WICI_MEGA_SHAPES(X)            \
-    X(128, MegaH4096, MegaF14336)      \
-    X(64, MegaH2048, MegaF8192)        \
-    X(128, MegaH5120, MegaF13824)      \
-    X(64, MegaSmall, MegaSmall)
+using MegaF12288 = GShape<6, 1, true>;    // Qwen3-8B widths: hidden 4096, ffn 12288
+// 8-bit block format: 16-element chunks per thread (NCH = ceil(K / 4096)), and
+// rows of q8_row_bytes(K) bytes per 32 KB slot: as many as fit, even where a
+// unit is a row pair
+using Q8H4096 = GShape<1, 6, true>;       // 6 x 4352 B
+using Q8F14336 = GShape<4, 2, false>;     // 2 x 15232 B; 896 chunks
+using Q8Small = GShape<1, 8, false>;      // 8 x <= 1904 B (K < 2048)
+using Q8F12288 = GShape<3, 2, true>;      // 2 x 13056 B
+// (head dim, bf16 shape K = hidden, bf16 shape K = ffn, 8-bit format, its shapes)
+#define WICI_MEGA_SHAPES(X)                                       \
+    X(128, MegaH4096, MegaF14336, false, MegaH4096, MegaF14336)   \
+    X(64, MegaH2048, MegaF8192, false, MegaH2048, MegaF8192)      \
+    X(128, MegaH5120, MegaF13824, false, MegaH5120, MegaF13824)   \
+    X(64, MegaSmall, MegaSmall, false, MegaSmall, MegaSmall)      \
+    X(128, MegaH4096, MegaF12288, false, MegaH4096, MegaF12288)   \
+    X(128, MegaH4096, MegaF14336, true, Q8H4096, Q8F14336)        \
+    X(128, MegaH4096, MegaF12288, true, Q8H4096, Q8F12288)        \
+    X(64, MegaSmall, MegaSmall, true, Q8Small, Q8Small)
 
 cudaError_t setup_kernels() {
     cudaError_t e;
-#define WICI_MEGA_ATTR(DD, SH, SF)                                                                  \
-    if ((e = cudaFuncSetAttribute(decode_step_kernel<DD, SH, SF>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
-                                  (int)kMegaSmem)) != cudaSuccess)                                    \
+#define WICI_MEGA_ATTR(DD, SH, SF, Q8, QH, QF)                                                        \
+    if ((e = cudaFuncSetAttribute(decode_step_kernel<DD, SH, SF, Q8, QH, QF>,                          \
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMegaSmem)) != cudaSuccess) \
         return e;
     WICI_MEGA_SHAPES(WICI_MEGA_ATTR)
 #undef WICI_MEGA_ATTR
@@ -1632,7 +1947,7 @@ cudaError_t enqueue_lm_head_argmax_raw(const uint16_t *W, const uint16_t *gain, 
 // ------------------------------------------------------- persistent decode: host
 typedef cudaError_t (*MegaLaunch)(const MegaArgs &, int grid, cudaStream_t);
 
-template <int D, class SH, class SF>
+template <int D, class SH, class SF, bool Q8, class QH, class QF>
 static cudaError_t launch_mega(const MegaArgs &a, int grid, cudaStream_t st) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
@@ -1644,12 +1959,20 @@ static cudaError_t launch_mega(const MegaArgs &a, int grid, cudaStream_t st) {
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, decode_step_kernel<D, SH, SF>, a);
+    return cudaLaunchKernelEx(&cfg, decode_step_kernel<D, SH, SF, Q8, QH, QF>, a);
 }
 
 template <class S>
 static bool shape_is(int K) {
     return gemv_nch(K) == S::NCH && gemv_rps(K) == S::RPS && ((K / 8) == S::NCH * kGemvConsumers) == S::FULL;
+}
+
+// 8-bit block rows: 16-element chunks, and S::RPS rows of the format in a slot
+template <class S>
+static bool q8_shape_is(int K) {
+    const int nch = (K / 16 + kGemvConsumers - 1) / kGemvConsumers;
+    return nch == S::NCH && ((K / 16) == nch * kGemvConsumers) == S::FULL &&
+           (size_t)S::RPS * q8_row_bytes((size_t)K) <= kMegaSlotBytes;
 }
 
 static MegaLaunch mega_launcher(const Plan &p) {
@@ -1662,12 +1985,14 @@ static MegaLaunch mega_launcher(const Plan &p) {
             const size_t o = st * (size_t)l;
             if (a.attn_norm != b.attn_norm + o || a.wqkv != b.wqkv + o || a.wo != b.wo + o ||
                 a.ffn_norm != b.ffn_norm + o || a.wgu != b.wgu + o || a.wd != b.wd + o ||
-                (p.cfg.qkv_bias && a.bqkv != b.bqkv + o))
+                (p.cfg.qkv_bias && a.bqkv != b.bqkv + o) || (p.qk_norm && (a.qn != b.qn + o || a.kn != b.kn + o)))
                 return nullptr;
         }
     }
-#define WICI_MEGA_PICK(DD, SH, SF) \
-    if (p.d == DD && shape_is<SH>(p.H) && shape_is<SF>(p.F)) return launch_mega<DD, SH, SF>;
+#define WICI_MEGA_PICK(DD, SH, SF, Q8, QH, QF)                                                       \
+    if (p.q8 == Q8 && p.d == DD && shape_is<SH>(p.H) && shape_is<SF>(p.F) &&                            \
+        (!Q8 || (q8_shape_is<QH>(p.H) && q8_shape_is<QF>(p.F))))                                        \
+        return launch_mega<DD, SH, SF, Q8, QH, QF>;
     WICI_MEGA_SHAPES(WICI_MEGA_PICK)
 #undef WICI_MEGA_PICK
     return nullptr;
@@ -1678,6 +2003,7 @@ bool decode_is_persistent(const Plan &p) { return mega_launcher(p) != nullptr; }
 static cudaError_t enqueue_mega(const Plan &p, const Bufs &b, cudaStream_t st, MegaLaunch fn) {
     MegaArgs a = {};
     a.W = b.W;
+    a.kraw = p.qk_norm ? b.kraw : nullptr;
     a.lstride = p.L > 1 ? p.layer[1].wqkv - p.layer[0].wqkv : 0;
     a.l0 = p.layer[0];
     a.w_embed = p.w_embed;
@@ -1703,8 +2029,8 @@ static cudaError_t enqueue_mega(const Plan &p, const Bufs &b, cudaStream_t st, M
     a.bias = p.cfg.qkv_bias;
     a.eps = p.cfg.rms_eps;
     a.qscale = 1.4426950408889634f / sqrtf((float)p.d);
-    cudaError_t e = cudaMemsetAsync(b.ctrl + CTRL_GRID_BAR, 0, sizeof(int), st);
-    if (e != cudaSuccess) return e;
+    // the grid-barrier counter is zero here: set at create, reset by the last CTA of
+    // every step, and by the host after a step that gave up
     return fn(a, grid, st);
 }
 

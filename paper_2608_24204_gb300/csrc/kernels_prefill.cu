@@ -4,6 +4,7 @@
 // and the causal attention on the tcgen05 attention kernel (attn_tc.cuh); the
 // kernels around them produce the tensor-core operands as bf16 hi/lo pairs.
 #include <cuda.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
@@ -74,6 +75,7 @@ struct PEpiQKV {  // packed QKV columns -> Q (three bf16 terms) and K/V pages (b
     const uint16_t *bias;
     int P, qdim, kvdim, d, nkv;
     size_t page_elems;
+    float *raw;      // qk_norm: q | k of row t land here as they are ([t][qdim + kvdim], natural order)
     __device__ void pair(int t, int c, float a, float b) const {
         if (bias) {
             a += bf16_to_f32(bias[c]);
@@ -82,7 +84,12 @@ struct PEpiQKV {  // packed QKV columns -> Q (three bf16 terms) and K/V pages (b
         const int pos = P + t;
         uint16_t *page = kv + (size_t)pages[pos / kPage] * page_elems;
         const int slot = pos % kPage;
-        if (c < qdim + kvdim) {
+        if (raw && c < qdim + kvdim) {
+            const int hd = c / d, i = (c % d) >> 1, half = d >> 1;
+            float *dst = raw + (size_t)t * (qdim + kvdim) + hd * d;
+            dst[i] = a;
+            dst[i + half] = b;
+        } else if (c < qdim + kvdim) {
             const int hd = c / d, i = (c % d) >> 1, half = d >> 1;
             const float2 cs = rope[(size_t)pos * half + i];
             const float ra = a * cs.x - b * cs.y;
@@ -122,7 +129,15 @@ struct PEpiQKV {  // packed QKV columns -> Q (three bf16 terms) and K/V pages (b
             float x[16];
 #pragma unroll
             for (int k = 0; k < 16; ++k) x[k] = v[g + k] + (bias ? bf16_to_f32(bias[c + k]) : 0.f);
-            if (c < qdim + kvdim) {
+            if (raw && c < qdim + kvdim) {
+                // 8 RoPE pairs (i0 + k, i0 + k + d/2) of one head, unnormalised
+                const int hd = c / d, i0 = (c % d) >> 1;
+                float *dst = raw + (size_t)t * (qdim + kvdim) + hd * d + i0;
+                *reinterpret_cast<float4 *>(dst) = make_float4(x[0], x[2], x[4], x[6]);
+                *reinterpret_cast<float4 *>(dst + 4) = make_float4(x[8], x[10], x[12], x[14]);
+                *reinterpret_cast<float4 *>(dst + half) = make_float4(x[1], x[3], x[5], x[7]);
+                *reinterpret_cast<float4 *>(dst + half + 4) = make_float4(x[9], x[11], x[13], x[15]);
+            } else if (c < qdim + kvdim) {
                 const int hd = c / d, i0 = (c % d) >> 1;
                 float ra[8], rb[8];
 #pragma unroll
@@ -246,6 +261,98 @@ struct PEpiSwiGLU {  // interleaved (gate, up) columns -> M[t][c/2] = silu(g) * 
     }
 };
 
+// ------------------------------------------------- Qwen3 q/k norm (prefill) --
+// One warp per (row t, head): the head of raw q (or k) RMS-normalised over
+// head_dim with its gain, RoPE at position P + t, then q as three bf16 terms in
+// Q[t] or k as bf16 in its page slot.  Lane l holds elements l*EPL ..; the RoPE
+// partner of element i < d/2 is i + d/2, in lane l + 16.
+template <int D>
+__global__ void qk_norm_rope_kernel(const float *raw, const uint16_t *qn, const uint16_t *kn, const float2 *rope,
+                                    Terms Q, uint16_t *kv, const int *pages, size_t page_elems, int P, int nq,
+                                    int nkv, float eps) {
+    constexpr int EPL = D / 32, HALF = D / 2;
+    const int t = blockIdx.x, lane = threadIdx.x & 31;
+    const int hd = blockIdx.y * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (hd >= nq + nkv) return;
+    const int qdim = nq * D, kvdim = nkv * D;
+    const float *src = raw + (size_t)t * (qdim + kvdim) + (size_t)hd * D + lane * EPL;
+    const uint16_t *gain = hd < nq ? qn : kn;
+    float v[EPL];
+    float ss = 0.f;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) {
+        v[e] = src[e];
+        ss = fmaf(v[e], v[e], ss);
+    }
+    const float rinv = 1.0f / sqrtf(warp_sum(ss) / (float)D + eps);
+    const int pos = P + t;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) v[e] = v[e] * rinv * bf16_to_f32(gain[lane * EPL + e]);
+    float r[EPL];
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) {
+        const float other = __shfl_xor_sync(0xffffffffu, v[e], 16);
+        const float2 cs = rope[(size_t)pos * HALF + (lane * EPL + e) % HALF];
+        r[e] = lane < 16 ? v[e] * cs.x - other * cs.y : v[e] * cs.x + other * cs.y;
+    }
+    if (hd < nq) {
+        const size_t o = (size_t)t * qdim + (size_t)hd * D + lane * EPL;
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) split_store(Q.p, o + e, r[e]);
+    } else {
+        uint16_t *kr = kv + (size_t)pages[pos / kPage] * page_elems + ((size_t)(hd - nq) * kPage + pos % kPage) * D +
+                       lane * EPL;
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) kr[e] = f32_to_bf16(r[e]);
+    }
+}
+
+// ------------------------------------------------ 8-bit block format (prefill) --
+// W[r][c] = d[r][c / 32] * code[r][c] of `rows` arena rows (int8 codes, then
+// the row's fp16 block scales), written as three bf16 terms of a
+// row-major [rows][K] matrix.  The product is exact in fp32 (at most 18
+// significant bits), and so is its split into three terms.  8 elements per
+// thread: one 8-byte code load, one scale, one 16-byte store per term.
+__global__ void q8_dequant_terms_kernel(const uint8_t *src, int rows, int K, const Terms out) {
+    const int per_row = K / 8;
+    const size_t rb = (size_t)K + (size_t)K / 16;
+    const long long n = (long long)rows * per_row;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        const long long r = i / per_row;
+        const int c = (int)(i - r * per_row);
+        const uint8_t *row = src + (size_t)r * rb;
+        const uint2 w = *reinterpret_cast<const uint2 *>(row + (size_t)c * 8);
+        const float d = __half2float(__ushort_as_half(*reinterpret_cast<const unsigned short *>(row + K + (c >> 2) * 2)));
+        uint32_t t[kTerms][4];
+#pragma unroll
+        for (int k = 0; k < 8; k += 2) {
+            const uint32_t word = k < 4 ? w.x : w.y;
+            const float a = d * (float)(int8_t)(word >> (8 * (k & 3)));
+            const float b = d * (float)(int8_t)(word >> (8 * ((k & 3) + 1)));
+            uint16_t ta[kTerms], tb[kTerms];
+            split_bf16x3(a, ta[0], ta[1], ta[2]);
+            split_bf16x3(b, tb[0], tb[1], tb[2]);
+#pragma unroll
+            for (int q = 0; q < kTerms; ++q) t[q][k >> 1] = (uint32_t)ta[q] | ((uint32_t)tb[q] << 16);
+        }
+        const size_t o = (size_t)r * K + (size_t)c * 8;
+#pragma unroll
+        for (int q = 0; q < kTerms; ++q)
+            *reinterpret_cast<uint4 *>(out.p[q] + o) = make_uint4(t[q][0], t[q][1], t[q][2], t[q][3]);
+    }
+}
+
+static cudaError_t dequant_terms(const Plan &p, const Bufs &b, const uint16_t *W, int rows, int K, cudaStream_t st,
+                                 LaunchHook *hook) {
+    const long long n = (long long)rows * (K / 8);
+    const int grid = (int)((n + 255) / 256 < 8 * p.num_sms ? (n + 255) / 256 : 8 * p.num_sms);
+    if (hook) hook->before("prefill_q8_dequant");
+    q8_dequant_terms_kernel<<<grid, 256, 0, st>>>(reinterpret_cast<const uint8_t *>(W), rows, K,
+                                                 Terms{{b.Wt[0], b.Wt[1], b.Wt[2]}});
+    if (hook) hook->after("prefill_q8_dequant");
+    return cudaGetLastError();
+}
+
 // --------------------------------------------------------------- RoPE table --
 __global__ void rope_table_kernel(float2 *rope, int n_pos, int half, double theta) {
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
@@ -332,11 +439,21 @@ const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
     m->bn_o = pick_bn(T, p.H, p.num_sms);
     m->bn_gu = pick_bn(T, 2 * p.F, p.num_sms);
     m->bn_d = pick_bn(T, p.H, p.num_sms);
-    m->wqkv.resize(p.L);
-    m->wo.resize(p.L);
-    m->wgu.resize(p.L);
-    m->wd.resize(p.L);
-    for (int l = 0; l < p.L; ++l) {
+    if (p.q8) {
+        // the 8-bit format: every GEMM reads the one dequantised matrix in the workspace
+        for (int t = 0; t < kTerms; ++t) {
+            ok = encode_2d(&m->wt_qkv[t], b.Wt[t], p.nqkv, p.H, m->bn_qkv) &&
+                 encode_2d(&m->wt_o[t], b.Wt[t], p.H, p.qdim, m->bn_o) &&
+                 encode_2d(&m->wt_gu[t], b.Wt[t], 2 * p.F, p.H, m->bn_gu) &&
+                 encode_2d(&m->wt_d[t], b.Wt[t], p.H, p.F, m->bn_d);
+            if (!ok) return "cuTensorMapEncodeTiled failed for a dequantised weight matrix";
+        }
+    }
+    m->wqkv.resize(p.q8 ? 0 : p.L);
+    m->wo.resize(p.q8 ? 0 : p.L);
+    m->wgu.resize(p.q8 ? 0 : p.L);
+    m->wd.resize(p.q8 ? 0 : p.L);
+    for (int l = 0; l < (p.q8 ? 0 : p.L); ++l) {
         const LayerOffsets &lo = p.layer[l];
         ok = encode_2d(&m->wqkv[l], b.W + lo.wqkv, p.nqkv, p.H, m->bn_qkv) &&
              encode_2d(&m->wo[l], b.W + lo.wo, p.H, p.qdim, m->bn_o) &&
@@ -350,12 +467,18 @@ const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
         const auto attr = [](const void *f, int bytes) {
             return cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) == cudaSuccess;
         };
-        if (!attr((const void *)gemm_tc_kernel<192, PEpiQKV>, s192) ||
-            !attr((const void *)gemm_tc_kernel<192, PEpiResidual>, s192) ||
-            !attr((const void *)gemm_tc_kernel<192, PEpiSwiGLU>, s192) ||
-            !attr((const void *)gemm_tc_kernel<128, PEpiQKV>, s128) ||
-            !attr((const void *)gemm_tc_kernel<128, PEpiResidual>, s128) ||
-            !attr((const void *)gemm_tc_kernel<128, PEpiSwiGLU>, s128) ||
+        if (!attr((const void *)gemm_tc_kernel<192, 1, PEpiQKV>, s192) ||
+            !attr((const void *)gemm_tc_kernel<192, 1, PEpiResidual>, s192) ||
+            !attr((const void *)gemm_tc_kernel<192, 1, PEpiSwiGLU>, s192) ||
+            !attr((const void *)gemm_tc_kernel<128, 1, PEpiQKV>, s128) ||
+            !attr((const void *)gemm_tc_kernel<128, 1, PEpiResidual>, s128) ||
+            !attr((const void *)gemm_tc_kernel<128, 1, PEpiSwiGLU>, s128) ||
+            !attr((const void *)gemm_tc_kernel<192, kTerms, PEpiQKV>, s192) ||
+            !attr((const void *)gemm_tc_kernel<192, kTerms, PEpiResidual>, s192) ||
+            !attr((const void *)gemm_tc_kernel<192, kTerms, PEpiSwiGLU>, s192) ||
+            !attr((const void *)gemm_tc_kernel<128, kTerms, PEpiQKV>, s128) ||
+            !attr((const void *)gemm_tc_kernel<128, kTerms, PEpiResidual>, s128) ||
+            !attr((const void *)gemm_tc_kernel<128, kTerms, PEpiSwiGLU>, s128) ||
             cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)(AttnSmem<128>::TOTAL + 1024)) != cudaSuccess ||
             cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -391,16 +514,27 @@ cudaError_t launch_attn_tc(const Plan &p, const Bufs &b, const PrefillMaps &mp, 
     return cudaGetLastError();
 }
 
+// the weight operand of one GEMM: one exact bf16 matrix, or three terms
+struct WOperand {
+    const CUtensorMap *w[kTerms];
+    int terms;
+};
+
 template <int BN, class Epi>
-static void launch_gemm(const Plan &p, const CUtensorMap *a, const CUtensorMap &w, int T, int N, int K, int *err,
+static void launch_gemm(const Plan &p, const CUtensorMap *a, const WOperand &w, int T, int N, int K, int *err,
                         const Epi &epi, cudaStream_t st) {
     const int tiles = ((T + TC_BM - 1) / TC_BM) * ((N + BN - 1) / BN);
     const int grid = tiles < p.num_sms ? tiles : p.num_sms;   // persistent: at most one CTA per SM
-    gemm_tc_kernel<BN, Epi><<<grid, TC_THREADS, TcTile<BN>::SMEM, st>>>(a[0], a[1], a[2], w, T, N, K, err, epi);
+    if (w.terms == 1)
+        gemm_tc_kernel<BN, 1, Epi><<<grid, TC_THREADS, TcTile<BN>::SMEM, st>>>(a[0], a[1], a[2], *w.w[0], *w.w[1],
+                                                                              *w.w[2], T, N, K, err, epi);
+    else
+        gemm_tc_kernel<BN, kTerms, Epi><<<grid, TC_THREADS, TcTile<BN>::SMEM, st>>>(
+            a[0], a[1], a[2], *w.w[0], *w.w[1], *w.w[2], T, N, K, err, epi);
 }
 
 template <class Epi>
-static cudaError_t gemm(const Plan &p, int bn, const CUtensorMap *a, const CUtensorMap &w, int T, int N, int K,
+static cudaError_t gemm(const Plan &p, int bn, const CUtensorMap *a, const WOperand &w, int T, int N, int K,
                         int *err, const Epi &epi, cudaStream_t st, LaunchHook *hook, const char *name) {
     if (hook) hook->before(name);
     if (bn == 128)
@@ -409,6 +543,19 @@ static cudaError_t gemm(const Plan &p, int bn, const CUtensorMap *a, const CUten
         launch_gemm<192>(p, a, w, T, N, K, err, epi, st);
     if (hook) hook->after(name);
     return cudaGetLastError();
+}
+
+// bf16: the layer's own matrix; 8-bit format: dequantise the layer's rows into
+// the workspace terms first (stream order makes the previous GEMM finish reading them)
+static cudaError_t weight_operand(const Plan &p, const Bufs &b, const CUtensorMap &bf16_map,
+                                  const CUtensorMap *terms, const uint16_t *rows, int n_rows, int K, cudaStream_t st,
+                                  LaunchHook *hook, WOperand *w) {
+    if (!p.q8) {
+        *w = WOperand{{&bf16_map, &bf16_map, &bf16_map}, 1};
+        return cudaSuccess;
+    }
+    *w = WOperand{{&terms[0], &terms[1], &terms[2]}, kTerms};
+    return dequant_terms(p, b, rows, n_rows, K, st, hook);
 }
 
 cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMaps &mp, cudaStream_t st, int P,
@@ -424,26 +571,53 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         const Terms A = {{b.A[0], b.A[1], b.A[2]}};
         rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.attn_norm, A, p.H, p.cfg.rms_eps);
         PEpiQKV eq = {{{b.Q[0], b.Q[1], b.Q[2]}}, kvl, b.pages, b.rope, p.cfg.qkv_bias ? b.W + lo.bqkv : nullptr, P, p.qdim,
-                      p.kvdim, p.d, p.nkv, p.kv_page_elems};
-        if ((e = gemm(p, mp.bn_qkv, mp.a, mp.wqkv[l], T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
+                      p.kvdim, p.d, p.nkv, p.kv_page_elems, p.qk_norm ? b.QKraw : nullptr};
+        WOperand w;
+        if ((e = weight_operand(p, b, p.q8 ? mp.wt_qkv[0] : mp.wqkv[l], mp.wt_qkv, b.W + lo.wqkv, p.nqkv, p.H, st,
+                                hook, &w)) != cudaSuccess)
             return e;
+        if ((e = gemm(p, mp.bn_qkv, mp.a, w, T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
+            return e;
+        if (p.qk_norm) {
+            // Qwen3 block: per-head q/k norm, then RoPE and the operand / page stores
+            const Terms Qt = {{b.Q[0], b.Q[1], b.Q[2]}};
+            const dim3 grid(T, (p.nq + p.nkv + 7) / 8);
+            if (hook) hook->before("prefill_qk_norm_rope");
+            if (p.d == 128)
+                qk_norm_rope_kernel<128><<<grid, 256, 0, st>>>(b.QKraw, b.W + lo.qn, b.W + lo.kn, b.rope, Qt, kvl,
+                                                               b.pages, p.kv_page_elems, P, p.nq, p.nkv, p.cfg.rms_eps);
+            else
+                qk_norm_rope_kernel<64><<<grid, 256, 0, st>>>(b.QKraw, b.W + lo.qn, b.W + lo.kn, b.rope, Qt, kvl,
+                                                              b.pages, p.kv_page_elems, P, p.nq, p.nkv, p.cfg.rms_eps);
+            if (hook) hook->after("prefill_qk_norm_rope");
+            if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        }
         // A5: causal attention over the cache (earlier chunks + this one), tensor cores
         if (hook) hook->before("prefill_attention");
         e = launch_attn_tc(p, b, mp, l, P, T, st);
         if (hook) hook->after("prefill_attention");
         if (e != cudaSuccess) return e;
         // A6: O projection + residual
-        if ((e = gemm(p, mp.bn_o, mp.o, mp.wo[l], T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
+        if ((e = weight_operand(p, b, p.q8 ? mp.wt_o[0] : mp.wo[l], mp.wt_o, b.W + lo.wo, p.H, p.qdim, st, hook,
+                                &w)) != cudaSuccess)
+            return e;
+        if ((e = gemm(p, mp.bn_o, mp.o, w, T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_o_proj")) != cudaSuccess)
             return e;
         // A7: RMSNorm + gate/up + SwiGLU
         rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.ffn_norm, A, p.H, p.cfg.rms_eps);
         const Terms M = {{b.M[0], b.M[1], b.M[2]}};
-        if ((e = gemm(p, mp.bn_gu, mp.a, mp.wgu[l], T, 2 * p.F, p.H, err, PEpiSwiGLU{M, p.F}, st, hook,
+        if ((e = weight_operand(p, b, p.q8 ? mp.wt_gu[0] : mp.wgu[l], mp.wt_gu, b.W + lo.wgu, 2 * p.F, p.H, st,
+                                hook, &w)) != cudaSuccess)
+            return e;
+        if ((e = gemm(p, mp.bn_gu, mp.a, w, T, 2 * p.F, p.H, err, PEpiSwiGLU{M, p.F}, st, hook,
                       "prefill_gate_up")) != cudaSuccess)
             return e;
         // A8: down projection + residual
-        if ((e = gemm(p, mp.bn_d, mp.m, mp.wd[l], T, p.H, p.F, err, PEpiResidual{b.X, p.H}, st, hook,
+        if ((e = weight_operand(p, b, p.q8 ? mp.wt_d[0] : mp.wd[l], mp.wt_d, b.W + lo.wd, p.H, p.F, st, hook,
+                                &w)) != cudaSuccess)
+            return e;
+        if ((e = gemm(p, mp.bn_d, mp.m, w, T, p.H, p.F, err, PEpiResidual{b.X, p.H}, st, hook,
                       "prefill_down")) != cudaSuccess)
             return e;
     }

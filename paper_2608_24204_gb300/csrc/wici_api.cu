@@ -78,6 +78,13 @@ const char *wici::make_plan(const wici_config *cfg, int num_sms, Plan *p) {
     if (!(c.rms_eps > 0.f) || !(c.rope_theta > 1.0)) return "rms_eps > 0 and rope_theta > 1 required";
     if (c.qkv_bias != 0 && c.qkv_bias != 1) return "qkv_bias must be 0 or 1";
     if (c.tied_embeddings != 0 && c.tied_embeddings != 1) return "tied_embeddings must be 0 or 1";
+    if (c.max_sms < 0) return "max_sms must be >= 0 (0: every SM)";
+    if (c.qk_norm != 0 && c.qk_norm != 1) return "qk_norm must be 0 or 1";
+    if (c.weight_format != WICI_WEIGHTS_BF16 && c.weight_format != WICI_WEIGHTS_Q8)
+        return "weight_format must be WICI_WEIGHTS_BF16 or WICI_WEIGHTS_Q8";
+    if (c.weight_format == WICI_WEIGHTS_Q8 &&
+        (c.hidden % 256 || c.ffn_dim % 256 || (c.n_q_heads * c.head_dim) % 256))
+        return "the 8-bit block format needs hidden, ffn_dim and n_q_heads*head_dim multiples of 256";
 
     Plan &P = *p;
     P.cfg = c;
@@ -88,22 +95,29 @@ const char *wici::make_plan(const wici_config *cfg, int num_sms, Plan *p) {
     P.max_pages = (c.max_tokens + kPage - 1) / kPage;
     P.max_chunk = c.max_chunk;
     P.num_sms = num_sms > 0 ? num_sms : 1;
+    if (c.max_sms > 0 && c.max_sms < P.num_sms) P.num_sms = c.max_sms;   // this tenant's SM share
+    P.q8 = c.weight_format == WICI_WEIGHTS_Q8;
+    P.qk_norm = c.qk_norm == 1;
 
     // weight arena: every tensor starts on a 128-byte boundary
     size_t off = 0;
     auto take = [&](size_t elems) { size_t o = off; off = align_up(off + elems, 64); return o; };
     const size_t H = P.H, F = P.F, V = P.V;
+    // a per-layer matrix [rows, K]: bf16, or rows of the 8-bit block format (in bf16 units)
+    auto mat = [&](size_t rows, size_t K) { return P.q8 ? rows * q8_row_bytes(K) / 2 : rows * K; };
     P.w_embed = take(V * H);
     P.layer.resize(P.L);
     for (int l = 0; l < P.L; ++l) {
         LayerOffsets &lo = P.layer[l];
         lo.attn_norm = take(H);
-        lo.wqkv = take((size_t)P.nqkv * H);
+        lo.wqkv = take(mat(P.nqkv, H));
         lo.bqkv = c.qkv_bias ? take((size_t)P.nqkv) : 0;
-        lo.wo = take(H * (size_t)P.qdim);
+        lo.qn = P.qk_norm ? take((size_t)P.d) : 0;
+        lo.kn = P.qk_norm ? take((size_t)P.d) : 0;
+        lo.wo = take(mat(H, P.qdim));
         lo.ffn_norm = take(H);
-        lo.wgu = take(2 * F * H);
-        lo.wd = take(H * F);
+        lo.wgu = take(mat(2 * F, H));
+        lo.wd = take(mat(H, F));
     }
     P.w_final_norm = take(H);
     P.w_lm = c.tied_embeddings ? P.w_embed : take(V * H);
@@ -138,6 +152,11 @@ const char *wici::make_plan(const wici_config *cfg, int num_sms, Plan *p) {
         P.ws_O[t] = ws(T * P.qdim * 2);
         P.ws_M[t] = ws(T * F * 2);
     }
+    P.wt_elems = 0;
+    for (size_t e : {(size_t)P.nqkv * H, H * (size_t)P.qdim, 2 * F * H, H * F}) P.wt_elems = e > P.wt_elems ? e : P.wt_elems;
+    for (int t = 0; t < kTerms; ++t) P.ws_Wt[t] = P.q8 ? ws(P.wt_elems * 2) : 0;
+    P.ws_kraw = P.qk_norm ? ws((size_t)P.kvdim * 4) : 0;
+    P.ws_QKraw = P.qk_norm ? ws(T * (size_t)(P.qdim + P.kvdim) * 4) : 0;
     P.ws_bytes = w;
     return nullptr;
 }
@@ -167,17 +186,20 @@ static Bufs make_bufs(const Plan &p, void *W, void *KV, void *WS) {
         b.A[t] = (uint16_t *)(ws + p.ws_A[t]);
         b.O[t] = (uint16_t *)(ws + p.ws_O[t]);
         b.M[t] = (uint16_t *)(ws + p.ws_M[t]);
+        b.Wt[t] = p.q8 ? (uint16_t *)(ws + p.ws_Wt[t]) : nullptr;
     }
+    b.kraw = p.qk_norm ? (float *)(ws + p.ws_kraw) : nullptr;
+    b.QKraw = p.qk_norm ? (float *)(ws + p.ws_QKraw) : nullptr;
     return b;
 }
 
 // canonical tensor index of a name, or -1; fills rows/cols expected and the layer
 struct TensorSlot { int kind; int layer; int64_t rows, cols; };
 enum { T_EMBED, T_FINAL_NORM, T_LM_HEAD, T_ATTN_NORM, T_WQ, T_WK, T_WV, T_BQ, T_BK, T_BV, T_WO,
-       T_FFN_NORM, T_WG, T_WU, T_WD, T_KINDS };
+       T_FFN_NORM, T_WG, T_WU, T_WD, T_QN, T_KN, T_KINDS };
 static const char *kLayerNames[] = {nullptr, nullptr, nullptr, "attn_norm", "wq", "wk", "wv", "bq",
-                                    "bk", "bv", "wo", "ffn_norm", "wg", "wu", "wd"};
-static const int kLayerKinds = 12;  // T_ATTN_NORM .. T_WD
+                                    "bk", "bv", "wo", "ffn_norm", "wg", "wu", "wd", "q_norm", "k_norm"};
+static const int kLayerKinds = 14;  // T_ATTN_NORM .. T_KN
 
 static bool parse_name(const Plan &p, const char *name, TensorSlot *s) {
     const int64_t H = p.H, F = p.F, V = p.V;
@@ -196,6 +218,7 @@ static bool parse_name(const Plan &p, const char *name, TensorSlot *s) {
     for (int k = T_ATTN_NORM; k < T_KINDS; ++k) {
         if (strcmp(leaf, kLayerNames[k])) continue;
         if ((k == T_BQ || k == T_BK || k == T_BV) && !p.cfg.qkv_bias) return false;
+        if ((k == T_QN || k == T_KN) && !p.qk_norm) return false;
         int64_t r = 0, c = 0;
         switch (k) {
             case T_ATTN_NORM: case T_FFN_NORM: r = 1; c = H; break;
@@ -206,11 +229,17 @@ static bool parse_name(const Plan &p, const char *name, TensorSlot *s) {
             case T_WO: r = H; c = p.qdim; break;
             case T_WG: case T_WU: r = F; c = H; break;
             case T_WD: r = H; c = F; break;
+            case T_QN: case T_KN: r = 1; c = p.d; break;
         }
         *s = {k, (int)l, r, c};
         return true;
     }
     return false;
+}
+
+static bool is_q8_kind(int kind) {
+    return kind == T_WQ || kind == T_WK || kind == T_WV || kind == T_WO || kind == T_WG || kind == T_WU ||
+           kind == T_WD;
 }
 
 static int slot_index(const Plan &p, const TensorSlot &s) {
@@ -277,12 +306,24 @@ int wici_create(const wici_config *cfg, void *cuda_stream, void *weight_dev, voi
         delete c;
         return fail(nullptr, WICI_E_ARG, "config: %s", m);
     }
+    if (c->plan.qk_norm && !decode_is_persistent(c->plan)) {
+        delete c;
+        return fail(nullptr, WICI_E_ARG,
+                    "config: the per-head q/k norm is built into the one-launch decode step, which needs "
+                    "n_q_heads * head_dim == hidden and an instantiated width");
+    }
+    if (c->plan.q8 && !decode_is_persistent(c->plan)) {
+        delete c;
+        return fail(nullptr, WICI_E_ARG,
+                    "config: the 8-bit block format is built for hidden 4096 / ffn 14336 (head_dim 128) and for "
+                    "hidden, ffn below 2048 (head_dim 64), with n_q_heads * head_dim == hidden");
+    }
     c->device = dev;
     c->stream = (cudaStream_t)cuda_stream;
     c->bufs = make_bufs(c->plan, weight_dev, kv_dev, workspace_dev);
     const Plan &p = c->plan;
     c->loaded.assign(3 + (size_t)p.L * kLayerKinds, 0);
-    c->n_required = 2 + (p.cfg.tied_embeddings ? 0 : 1) + p.L * (p.cfg.qkv_bias ? 12 : 9);
+    c->n_required = 2 + (p.cfg.tied_embeddings ? 0 : 1) + p.L * (9 + (p.cfg.qkv_bias ? 3 : 0) + (p.qk_norm ? 2 : 0));
     int rc = WICI_OK;
     do {
         if ((e = setup_kernels()) != cudaSuccess) break;
@@ -333,6 +374,9 @@ int wici_load_weights(wici_ctx *c, const wici_tensor *t, int32_t n) {
         TensorSlot s;
         if (!t[i].name || !t[i].data) return fail(c, WICI_E_ARG, "tensor %d: null name or data", i);
         if (!parse_name(p, t[i].name, &s)) return fail(c, WICI_E_ARG, "unknown tensor name '%s'", t[i].name);
+        if (p.q8 && is_q8_kind(s.kind))
+            return fail(c, WICI_E_ARG, "'%s' is in the 8-bit block format here: load it with wici_load_weights_q8",
+                        t[i].name);
         if (t[i].rows != s.rows || t[i].cols != s.cols)
             return fail(c, WICI_E_ARG, "tensor '%s': shape [%lld, %lld], expected [%lld, %lld]", t[i].name,
                         (long long)t[i].rows, (long long)t[i].cols, (long long)s.rows, (long long)s.cols);
@@ -376,8 +420,88 @@ int wici_load_weights(wici_ctx *c, const wici_tensor *t, int32_t n) {
                 case T_WD:
                     e = cudaMemcpyAsync(W + lo.wd, src, (size_t)H * p.F * 2, cudaMemcpyDefault, c->stream);
                     break;
+                case T_QN: e = cudaMemcpyAsync(W + lo.qn, src, (size_t)p.d * 2, cudaMemcpyDefault, c->stream); break;
+                case T_KN: e = cudaMemcpyAsync(W + lo.kn, src, (size_t)p.d * 2, cudaMemcpyDefault, c->stream); break;
             }
         }
+        if (e != cudaSuccess) return fail(c, WICI_E_CUDA, "copy of '%s': %s", t[i].name, cudaGetErrorString(e));
+        const int si = slot_index(p, s);
+        if (!c->loaded[si]) {
+            c->loaded[si] = 1;
+            ++c->n_loaded;
+        }
+    }
+    CUDA_TRY(c, cudaStreamSynchronize(c->stream));
+    return WICI_OK;
+}
+
+// Rows of one matrix in the 8-bit block format: codes and scales of source row
+// r go to arena row dst_row(r) (codes first, then the K/32 scales); the RoPE
+// pairing of wq/wk and the gate/up interleaving are the bf16 loader's.
+static cudaError_t copy_q8_rows(uint8_t *dst, size_t drow_bytes, int dst_step, const uint8_t *codes,
+                                const uint8_t *scales, int64_t rows, int64_t K, cudaStream_t st) {
+    cudaError_t e = cudaMemcpy2DAsync(dst, drow_bytes * dst_step, codes, (size_t)K, (size_t)K, (size_t)rows,
+                                      cudaMemcpyDefault, st);
+    if (e != cudaSuccess) return e;
+    return cudaMemcpy2DAsync(dst + K, drow_bytes * dst_step, scales, (size_t)K / 16, (size_t)K / 16, (size_t)rows,
+                             cudaMemcpyDefault, st);
+}
+
+static cudaError_t load_q8(const Plan &p, uint16_t *W, const TensorSlot &s, const wici_q8_tensor &t,
+                           cudaStream_t st) {
+    const LayerOffsets &lo = p.layer[s.layer];
+    const int64_t K = s.cols;
+    const size_t rb = q8_row_bytes((size_t)K);
+    uint8_t *base = nullptr;   // the matrix's first arena row
+    int step = 1;              // arena rows per source row
+    int64_t row0 = 0;          // first arena row of this tensor inside `base`
+    switch (s.kind) {
+        case T_WQ: base = (uint8_t *)(W + lo.wqkv); break;
+        case T_WK: base = (uint8_t *)(W + lo.wqkv); row0 = p.qdim; break;
+        case T_WV: base = (uint8_t *)(W + lo.wqkv); row0 = p.qdim + p.kvdim; break;
+        case T_WO: base = (uint8_t *)(W + lo.wo); break;
+        case T_WG: base = (uint8_t *)(W + lo.wgu); step = 2; break;
+        case T_WU: base = (uint8_t *)(W + lo.wgu); step = 2; row0 = 1; break;
+        case T_WD: base = (uint8_t *)(W + lo.wd); break;
+    }
+    const uint8_t *codes = (const uint8_t *)t.codes, *scales = (const uint8_t *)t.scales;
+    cudaError_t e = cudaSuccess;
+    if (s.kind == T_WQ || s.kind == T_WK) {
+        // per head: rows i and i + d/2 become adjacent arena rows 2i, 2i + 1
+        const int heads = (int)(s.rows / p.d), half = p.d / 2;
+        for (int h = 0; h < heads && e == cudaSuccess; ++h) {
+            uint8_t *dst = base + (size_t)(row0 + (int64_t)h * p.d) * rb;
+            const size_t sr = (size_t)h * p.d;
+            e = copy_q8_rows(dst, rb, 2, codes + sr * K, scales + sr * (K / 16), half, K, st);
+            if (e == cudaSuccess)
+                e = copy_q8_rows(dst + rb, rb, 2, codes + (sr + half) * K, scales + (sr + half) * (K / 16), half, K,
+                                 st);
+        }
+    } else {
+        e = copy_q8_rows(base + (size_t)row0 * rb, rb, step, codes, scales, s.rows, K, st);
+    }
+    return e;
+}
+
+int wici_load_weights_q8(wici_ctx *c, const wici_q8_tensor *t, int32_t n) {
+    if (!c) return fail(nullptr, WICI_E_ARG, "null context");
+    if (!t || n < 0) return fail(c, WICI_E_ARG, "bad tensor list");
+    const Plan &p = c->plan;
+    if (!p.q8) return fail(c, WICI_E_ARG, "the context holds bf16 matrices (weight_format = WICI_WEIGHTS_BF16)");
+    for (int i = 0; i < n; ++i) {
+        TensorSlot s;
+        if (!t[i].name || !t[i].codes || !t[i].scales)
+            return fail(c, WICI_E_ARG, "tensor %d: null name, codes or scales", i);
+        if (!parse_name(p, t[i].name, &s) || !is_q8_kind(s.kind))
+            return fail(c, WICI_E_ARG, "'%s' is not a per-layer matrix of the 8-bit format", t[i].name);
+        if (t[i].rows != s.rows || t[i].cols != s.cols)
+            return fail(c, WICI_E_ARG, "tensor '%s': shape [%lld, %lld], expected [%lld, %lld]", t[i].name,
+                        (long long)t[i].rows, (long long)t[i].cols, (long long)s.rows, (long long)s.cols);
+    }
+    for (int i = 0; i < n; ++i) {
+        TensorSlot s;
+        parse_name(p, t[i].name, &s);
+        cudaError_t e = load_q8(p, c->bufs.W, s, t[i], c->stream);
         if (e != cudaSuccess) return fail(c, WICI_E_CUDA, "copy of '%s': %s", t[i].name, cudaGetErrorString(e));
         const int si = slot_index(p, s);
         if (!c->loaded[si]) {
@@ -407,6 +531,7 @@ static int finish_call(wici_ctx *c, int32_t new_kv_len, int32_t *token_out) {
         cudaMemcpyAsync(c->bufs.ctrl + CTRL_ERR, c->pinned + 3, sizeof(int), cudaMemcpyHostToDevice, c->stream);
         cudaMemcpyAsync(c->bufs.ctrl + CTRL_POS, c->pinned + 4, sizeof(int), cudaMemcpyHostToDevice, c->stream);
         cudaMemsetAsync(c->bufs.ctrl + CTRL_LM_TICKET, 0, sizeof(int), c->stream);
+        cudaMemsetAsync(c->bufs.ctrl + CTRL_GRID_BAR, 0, sizeof(int), c->stream);
         cudaMemsetAsync(c->bufs.ctrl + CTRL_ATTN_TICKET0, 0, 64 * sizeof(int), c->stream);
         cudaStreamSynchronize(c->stream);
         return fail(c, WICI_E_TIMEOUT, "a device-side wait gave up (site %d)", errw);

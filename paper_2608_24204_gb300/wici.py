@@ -20,7 +20,8 @@ STATUS_NAMES = {0: "WICI_OK", -1: "WICI_E_ARG", -2: "WICI_E_STATE", -3: "WICI_E_
                 -4: "WICI_E_CUDA", -5: "WICI_E_TIMEOUT"}
 
 # the entry points declared in include/wici.h
-EXPORTS = ("wici_get_sizes", "wici_create", "wici_load_weights", "wici_prefill", "wici_decode_step",
+EXPORTS = ("wici_get_sizes", "wici_create", "wici_load_weights", "wici_load_weights_q8", "wici_prefill",
+           "wici_decode_step",
            "wici_decode", "wici_reset", "wici_set_page_table", "wici_kv_len", "wici_last_error",
            "wici_profile_decode", "wici_check_bounded_wait", "wici_destroy", "wici_lm_head_argmax_noalloc")
 
@@ -30,7 +31,10 @@ class wici_config(ctypes.Structure):
                 ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("ffn_dim", ctypes.c_int32),
                 ("vocab", ctypes.c_int32), ("max_tokens", ctypes.c_int32), ("max_chunk", ctypes.c_int32),
                 ("page_tokens", ctypes.c_int32), ("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_double),
-                ("tied_embeddings", ctypes.c_int32), ("qkv_bias", ctypes.c_int32)]
+                ("tied_embeddings", ctypes.c_int32), ("qkv_bias", ctypes.c_int32),
+                ("weight_format", ctypes.c_int32), ("qk_norm", ctypes.c_int32), ("max_sms", ctypes.c_int32)]
+
+WICI_WEIGHTS_BF16, WICI_WEIGHTS_Q8 = 0, 1
 
 
 class wici_sizes(ctypes.Structure):
@@ -41,6 +45,11 @@ class wici_sizes(ctypes.Structure):
 class wici_tensor(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char_p), ("data", ctypes.c_void_p), ("rows", ctypes.c_int64),
                 ("cols", ctypes.c_int64), ("on_device", ctypes.c_int32)]
+
+
+class wici_q8_tensor(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char_p), ("codes", ctypes.c_void_p), ("scales", ctypes.c_void_p),
+                ("rows", ctypes.c_int64), ("cols", ctypes.c_int64), ("on_device", ctypes.c_int32)]
 
 
 _lib = None
@@ -58,6 +67,7 @@ def lib():
         L.wici_get_sizes.argtypes = [P(wici_config), P(wici_sizes)]
         L.wici_create.argtypes = [P(wici_config), vp, vp, vp, vp, P(vp)]
         L.wici_load_weights.argtypes = [vp, P(wici_tensor), i32]
+        L.wici_load_weights_q8.argtypes = [vp, P(wici_q8_tensor), i32]
         L.wici_prefill.argtypes = [vp, P(i32), i32, P(ctypes.c_float), P(i32)]
         L.wici_decode_step.argtypes = [vp, i32, P(ctypes.c_float), P(i32)]
         L.wici_decode.argtypes = [vp, i32, i32, P(i32)]
@@ -72,7 +82,8 @@ def lib():
         L.wici_destroy.argtypes = [vp]
         L.wici_destroy.restype = None
         L.wici_lm_head_argmax_noalloc.argtypes = [vp, vp, vp, vp, i32, i32, ctypes.c_float, vp, vp]
-        for name in ("wici_get_sizes", "wici_create", "wici_load_weights", "wici_prefill", "wici_decode_step",
+        for name in ("wici_get_sizes", "wici_create", "wici_load_weights", "wici_load_weights_q8", "wici_prefill",
+                     "wici_decode_step",
                      "wici_decode", "wici_reset", "wici_set_page_table", "wici_profile_decode",
                      "wici_check_bounded_wait", "wici_lm_head_argmax_noalloc"):
             getattr(L, name).restype = ctypes.c_int
@@ -92,11 +103,14 @@ def _check(rc, ctx=None):
     return rc
 
 
-def make_config(cfg, max_tokens: int, max_chunk: int | None = None) -> wici_config:
+def make_config(cfg, max_tokens: int, max_chunk: int | None = None, q8: bool = False,
+                max_sms: int = 0) -> wici_config:
     """wici_config from a gen.ModelConfig-like object."""
     return wici_config(cfg.n_layers, cfg.hidden, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.ffn_dim,
                        cfg.vocab, max_tokens, min(max_chunk or cfg.max_chunk, max_tokens), 16, cfg.rms_eps,
-                       cfg.rope_theta, int(cfg.tied_embeddings), int(cfg.qkv_bias))
+                       cfg.rope_theta, int(cfg.tied_embeddings), int(cfg.qkv_bias),
+                       WICI_WEIGHTS_Q8 if q8 else WICI_WEIGHTS_BF16, int(getattr(cfg, "qk_norm", False)),
+                       max_sms)
 
 
 # ---------------------------------------------------------------- thin wrappers
@@ -125,6 +139,19 @@ def wici_load_weights(ctx, tensors) -> None:
         arr.append(wici_tensor(name.encode(), ptr, rows, cols, dev))
     tarr = (wici_tensor * len(arr))(*arr)
     _check(lib().wici_load_weights(ctx, tarr, len(arr)), ctx)
+
+
+def wici_load_weights_q8(ctx, tensors) -> None:
+    """tensors: iterable of (name, codes int8 [rows, cols], scales fp16 bits uint16 [rows, cols/32]) host arrays."""
+    keep, arr = [], []
+    for name, codes, scales in tensors:
+        codes = np.ascontiguousarray(codes, np.int8)
+        scales = np.ascontiguousarray(scales, np.uint16)
+        keep += [codes, scales]
+        arr.append(wici_q8_tensor(name.encode(), codes.ctypes.data, scales.ctypes.data, codes.shape[0],
+                                  codes.shape[1], 0))
+    tarr = (wici_q8_tensor * len(arr))(*arr)
+    _check(lib().wici_load_weights_q8(ctx, tarr, len(arr)), ctx)
 
 
 def _i32p(a):
@@ -198,13 +225,14 @@ def wici_lm_head_argmax_noalloc(stream: int, lm_head_dev: int, norm_gain_dev: in
 class WiciModel:
     """Owns torch-allocated device buffers and one context on the current device."""
 
-    def __init__(self, cfg, max_tokens: int | None = None, max_chunk: int | None = None, stream=None):
+    def __init__(self, cfg, max_tokens: int | None = None, max_chunk: int | None = None, stream=None,
+                 q8: bool = False, max_sms: int = 0):
         import torch
         if not torch.cuda.is_available():
             raise RuntimeError("WiciModel needs a CUDA device")
         self.cfg = cfg
         self.max_tokens = max_tokens or cfg.total_tokens
-        self.ccfg = make_config(cfg, self.max_tokens, max_chunk)
+        self.ccfg = make_config(cfg, self.max_tokens, max_chunk, q8, max_sms)
         sizes = wici_get_sizes(self.ccfg)
         self.sizes = sizes
 
@@ -221,12 +249,20 @@ class WiciModel:
         self.ctx = wici_create(self.ccfg, self.stream.cuda_stream, aligned(self._w), aligned(self._kv),
                                aligned(self._ws))
 
-    def load(self, weights: dict) -> "WiciModel":
+    def load(self, weights: dict, q8_weights: dict | None = None) -> "WiciModel":
+        """bf16 tensors {name: uint16 [rows, cols]}; with the 8-bit format, the
+        per-layer matrices come as q8_weights {name: (codes, scales)} and the
+        bf16 dict's entries of the same names are skipped."""
+        q8_weights = q8_weights or {}
         items = []
         for name, arr in weights.items():
+            if name in q8_weights:
+                continue
             r, c = arr.shape
             items.append((name, arr, r, c))
         wici_load_weights(self.ctx, items)
+        if q8_weights:
+            wici_load_weights_q8(self.ctx, [(n, c, s) for n, (c, s) in q8_weights.items()])
         return self
 
     def prefill(self, tokens, logits: bool = False):

@@ -26,7 +26,7 @@ def declared_entry_points():
 
 def test_library_exports_every_declared_entry_point():
     names = declared_entry_points()
-    assert len(names) == 14
+    assert len(names) == 15
     L = wici.lib()
     for n in names:
         assert hasattr(L, n), n
@@ -43,6 +43,28 @@ def test_sizes_match_the_packed_layout():
     tied = wici.wici_get_sizes(wici.make_config(gen.LLAMA_1B, 640))
     p1 = sum(r * c for _, (r, c), _ in gen.tensor_specs(gen.LLAMA_1B))
     assert p1 * 2 <= tied.weight_bytes <= p1 * 2 + 1_000_000   # the LM head aliases the embedding
+
+
+def test_q8_sizes_hold_codes_and_block_scales():
+    # the seven per-layer matrices at 17/16 bytes per parameter (codes + one fp16
+    # scale per 32), everything else bf16; the prefill workspace adds one matrix
+    # (the largest, gate|up) as three bf16 terms
+    cfg = gen.LLAMA_8B
+    b = wici.wici_get_sizes(wici.make_config(cfg, max_tokens=1296, max_chunk=1024))
+    q = wici.wici_get_sizes(wici.make_config(cfg, max_tokens=1296, max_chunk=1024, q8=True))
+    per_layer = sum(r * c for n, (r, c), _ in gen.tensor_specs(cfg)
+                    if n.startswith("layers.0.") and n.split(".")[-1] in ("wq", "wk", "wv", "wo", "wg", "wu", "wd"))
+    saved = cfg.n_layers * per_layer * (2 - 17 / 16)
+    assert abs((b.weight_bytes - q.weight_bytes) - saved) < 1_000_000
+    assert q.workspace_bytes - b.workspace_bytes >= 3 * 2 * (2 * cfg.ffn_dim * cfg.hidden)
+    assert q.kv_bytes == b.kv_bytes
+
+
+def test_q8_rejects_widths_that_are_not_multiples_of_256():
+    with pytest.raises(wici.WiciError) as e:
+        wici.wici_get_sizes(wici.make_config(gen.TINY, 64, q8=True))      # ffn 688
+    assert e.value.status == wici.WICI_E_ARG and "256" in str(e.value)
+    wici.wici_get_sizes(wici.make_config(gen.TINY.with_(ffn_dim=768), 64, q8=True))
 
 
 @pytest.mark.parametrize("field,value", [("head_dim", 96), ("n_kv_heads", 3), ("page_tokens", 32),

@@ -110,6 +110,8 @@ def _full(cfg, decode_steps, max_chunk=None):
     stats = {}
     run_teacher_forced(model, ref, [prompt], decode_steps, stats)
     model.close()
+    print(f"\n{cfg.name}: {len(stats['max_abs'])} positions; max-abs {max(stats['max_abs']):.3e} "
+          f"(prefill {stats['max_abs'][0]:.3e}), rel-L2 {max(stats['rel_l2']):.3e}; near ties {stats.get('near_ties', 0)}")
     return stats
 
 

@@ -293,8 +293,13 @@ def _torch_restatement(cfg, w, tokens, mats=None):
     for l in range(cfg.n_layers):
         p = f"layers.{l}."
         h = F.rms_norm(x, (cfg.hidden,), W(p + "attn_norm")[0], eps=cfg.rms_eps)
-        q = rope(F.linear(h, W(p + "wq"), B(p + "bq")).view(T, nq, d))
-        k = bf16(rope(F.linear(h, W(p + "wk"), B(p + "bk")).view(T, nkv, d)))
+        q = F.linear(h, W(p + "wq"), B(p + "bq")).view(T, nq, d)
+        k = F.linear(h, W(p + "wk"), B(p + "bk")).view(T, nkv, d)
+        if cfg.qk_norm:
+            q = F.rms_norm(q, (d,), W(p + "q_norm")[0], eps=cfg.rms_eps)
+            k = F.rms_norm(k, (d,), W(p + "k_norm")[0], eps=cfg.rms_eps)
+        q = rope(q)
+        k = bf16(rope(k))
         v = bf16(F.linear(h, W(p + "wv"), B(p + "bv")).view(T, nkv, d))
         k = k.repeat_interleave(nq // nkv, dim=1)
         v = v.repeat_interleave(nq // nkv, dim=1)
@@ -326,6 +331,43 @@ def test_one_wide_layer_matches_torch_restatement():
     prompt = gen.make_prompt(cfg, 24, seed=1)
     got, _ = oracle.OracleModel(cfg, w, max_tokens=32).prefill(prompt)
     np.testing.assert_allclose(got, _torch_restatement(cfg, w, prompt), rtol=0, atol=1e-6)
+
+
+TINY_QK = gen.TINY.with_(name="tiny-qk", qk_norm=True, rope_theta=1e6, rms_eps=1e-6)
+
+
+def test_qk_norm_model_matches_independent_torch_restatement():
+    cfg = TINY_QK
+    w = _tiny_weights(cfg)
+    assert "layers.0.q_norm" in w and w["layers.0.q_norm"].shape == (1, cfg.head_dim)
+    prompt = gen.make_prompt(cfg, 24, seed=1)
+    got, _ = oracle.OracleModel(cfg, w, max_tokens=32).prefill(prompt)
+    want = _torch_restatement(cfg, w, prompt)
+    np.testing.assert_allclose(got, want, rtol=1e-6, atol=1e-6)
+
+
+def test_qk_norm_makes_logits_blind_to_the_scale_of_wq_and_wk():
+    # per-head RMSNorm of q and k removes any scale of their projections (up to
+    # eps and the bf16 rounding of the stored keys): Wq x 2 and Wk x 4 leave the
+    # logits unchanged, while without the norms every score grows eightfold
+    def run(cfg, w):
+        return oracle.OracleModel(cfg, w, max_tokens=32).prefill(gen.make_prompt(cfg, 20, seed=3))[0]
+
+    def rescaled(w, cfg):
+        w = dict(w)
+        for l in range(cfg.n_layers):
+            for name, f in (("wq", 2.0), ("wk", 4.0)):
+                v = L.bf16_bits_to_f64(w[f"layers.{l}.{name}"]) * f        # exact in bf16
+                w[f"layers.{l}.{name}"] = (v.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+        return w
+
+    w = _tiny_weights(TINY_QK)
+    base, moved = run(TINY_QK, w), run(TINY_QK, rescaled(w, TINY_QK))
+    scale = np.abs(base).max()
+    np.testing.assert_allclose(moved, base, rtol=0, atol=2e-3 * scale)
+    plain = gen.TINY.with_(name="tiny-qk-off", rope_theta=1e6, rms_eps=1e-6)
+    wp = {k: v for k, v in w.items() if "q_norm" not in k and "k_norm" not in k}
+    assert np.abs(run(plain, rescaled(wp, plain)) - run(plain, wp)).max() > 5e-2 * scale
 
 
 def test_qkv_bias_is_added_before_rope():
