@@ -13,8 +13,10 @@ peak), `agentic`: the agentic long-context workload at the same shape
 (4 turns of a 2048-token chunk plus 64 decode steps, 8448 cached), timed after
 the K requests, with its four chunk prefills in aggregate against the bf16 peak,
 `multi_tenant`: a 1B-shaped and the 8B-shaped model decoding at the same
-time on SM shares of one GPU, per-tenant tokens/s, and `q8`: the 8B request
-with its per-layer matrices in the 8-bit block format.
+time on SM shares of one GPU, per-tenant tokens/s, `q8`: the 8B request
+with its per-layer matrices in the 8-bit block format, and `cnn_train`: the
+paper's CNN-training sample (a 3x3 stride-2 convolution layer on 4 x 1024 x
+224 x 224, forward and both gradients) against the bf16 tensor peak.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -286,6 +288,56 @@ def measure_q8(weights_8b, WiciModel, torch, pk, runs: int = 3):
             "ttft_ms": statistics.median(ttft), "runs": runs}
 
 
+def measure_cnn_train(torch, pk, runs: int = 3):
+    """The CNN-training sample (Sec. 5.4): one 3x3 stride-2 convolution layer on
+    a 4 x 1024 x 224 x 224 input with 1024 output channels, forward plus the data
+    and filter gradients, each timed with CUDA events (median of `runs` after one
+    untimed run) against the bf16 tensor peak (each is 2 N P Q K C 9 FLOPs)."""
+    from gen import conv as gc
+    from paper_2608_24204_gb300 import wici
+    s = gc.CNN_SAMPLE
+    x, w, dy = gc.make_conv_inputs(s)
+    dev = lambda a: torch.from_numpy(a.view(np.int16)).cuda()  # noqa: E731
+    xd, wd, dyd = dev(x), dev(w), dev(dy)
+    del x, w, dy
+    shape = wici.wici_conv_shape(s.n, s.c, s.h, s.w, s.k)
+    ws = torch.zeros(wici.wici_conv_workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    y = torch.empty((s.n, s.p, s.q, s.k), device="cuda")
+    dx = torch.empty((s.n, s.h, s.w, s.c), device="cuda")
+    dw = torch.empty((s.k, 3, 3, s.c), device="cuda")
+    st = torch.cuda.current_stream()
+    calls = {"forward": lambda: wici.wici_conv_forward(st.cuda_stream, shape, xd.data_ptr(), wd.data_ptr(),
+                                                       y.data_ptr(), ws.data_ptr()),
+             "data_gradient": lambda: wici.wici_conv_backward_data(st.cuda_stream, shape, dyd.data_ptr(),
+                                                                   wd.data_ptr(), dx.data_ptr(), ws.data_ptr()),
+             "filter_gradient": lambda: wici.wici_conv_backward_filter(st.cuda_stream, shape, xd.data_ptr(),
+                                                                       dyd.data_ptr(), dw.data_ptr(), ws.data_ptr())}
+    ms = {k: [] for k in calls}
+    for r in range(runs + 1):
+        for k, f in calls.items():
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            f()
+            e1.record(st)
+            e1.synchronize()
+            if r > 0:
+                ms[k].append(e0.elapsed_time(e1))
+    wici.wici_conv_status(st.cuda_stream, ws.data_ptr())
+    fl = s.flops()
+    out = {"workload": f"conv 3x3 stride 2 pad 1: x {s.n}x{s.c}x{s.h}x{s.w} (channels last, bf16), {s.k} filters; "
+                       "forward, data gradient, filter gradient; fp32 outputs",
+           "flops_each": fl, "peak": pk["bf16_tflops"], "unit": "TFLOP/s"}
+    tot = 0.0
+    for k in calls:
+        m = statistics.median(ms[k])
+        tot += m
+        out[k] = {"ms": m, "tflops": fl / (m / 1000.0) / 1e12, "frac": fl / (m / 1000.0) / 1e12 / pk["bf16_tflops"]}
+    out["step_ms"] = tot
+    out["step_tflops"] = 3 * fl / (tot / 1000.0) / 1e12
+    out["step_frac"] = out["step_tflops"] / pk["bf16_tflops"]
+    return out
+
+
 def measure_multi_tenant(weights_8b, WiciModel, torch, steps: int = 256):
     """Two tenants on one GPU, as in the paper's two-client microbenchmark: a
     Llama-3.2-1B-shaped model (512-token prompt) and the Llama-3-8B-shaped one
@@ -502,13 +554,14 @@ def run_ours(args):
                         "flops_per_prefill": pf_flops, "ttft_ms": ttft_med, "peak_source": pk["source"],
                         "what": f"algorithmic FLOPs of the {PROMPT}-token prefill / TTFT (CUDA events)"}
 
-    agentic = tenants = q8 = None
+    agentic = tenants = q8 = cnn = None
     if not args.no_agentic and CFG.n_layers == gen.LLAMA_8B.n_layers:
         model.close()
         model = None
         agentic = measure_agentic(weights, WiciModel, torch, pk)
         tenants = measure_multi_tenant(weights, WiciModel, torch)
         q8 = measure_q8(weights, WiciModel, torch, pk)
+        cnn = measure_cnn_train(torch, pk)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -534,7 +587,7 @@ def run_ours(args):
             "bytes_per_token": bytes_tok,
             "prefill_tflops": pf_tf,
             "roofline": roofline, "prefill_roofline": prefill_roofline, "agentic": agentic,
-            "multi_tenant": tenants, "q8": q8,
+            "multi_tenant": tenants, "q8": q8, "cnn_train": cnn,
             "kernels": kernel_share, "cpu_baseline": cpu,
             "e2e": {"value": e2e_val, "unit": "tok/s", "h2d_bytes_per_step": PROMPT * 4,
                     "d2h_bytes_per_step": (DECODE + 1) * 4, "ttft_ms": statistics.median(e2e_ttft),
@@ -560,7 +613,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-agentic", action="store_true",
-                    help="skip the agentic, two-tenant and 8-bit-format measurements")
+                    help="skip the agentic, two-tenant, 8-bit-format and CNN measurements")
     ap.add_argument("--quick", action="store_true", help="profiling run: timed requests only")
     ap.add_argument("--decode-steps", type=int, default=0, help="profiling run: decode steps per request")
     ap.add_argument("--layers", type=int, default=0, help="profiling run: fewer layers (small ncu case)")

@@ -242,6 +242,44 @@ int wici_lm_head_argmax_noalloc(void *cuda_stream, const void *lm_head_dev, cons
                                 const float *x_dev, int32_t hidden, int32_t vocab, float rms_eps,
                                 float *logits_dev, int32_t *token_dev);
 
+/* ---------------------------------------------------------------------------
+ * CNN-training sample (Sec. 5.4, "Multiple applications": NVIDIA's CNN training
+ * sample, input 4 x 1024 x 224 x 224, 3x3 filter, stride 2).  One convolution
+ * layer, 3x3, stride 2, zero padding 1 (readings: padding 1, no bias), forward
+ * and the two gradients of backpropagation, on the tensor cores.  Channels last,
+ * row-major, device pointers, 16-byte aligned:
+ *   x  bf16 [n][h][w][c]      w  bf16 [k][3][3][c]     dy bf16 [n][h/2][w/2][k]
+ *   y  fp32 [n][h/2][w/2][k]  dx fp32 [n][h][w][c]     dw fp32 [k][3][3][c]
+ * Constraints: c and k multiples of 256; h and w even; n >= 1 (else WICI_E_ARG,
+ * message in wici_last_error(NULL)).  Each call is enqueued on cuda_stream and
+ * returns without synchronising; `workspace` (wici_conv_workspace_bytes, zeroed
+ * once by the caller before its first use) holds the error word and, for the
+ * data gradient, the transposed filter.  Calls sharing a workspace must be
+ * ordered on one stream. */
+typedef struct wici_conv_shape {
+    int32_t n, c, h, w, k;
+} wici_conv_shape;
+
+/* Bytes of the workspace for `s`. */
+int wici_conv_workspace_bytes(const wici_conv_shape *s, size_t *bytes);
+
+/* y[pix][k] = sum over taps and c of x at (2p + r - 1, 2q + s - 1) times w[k][r][s][c]. */
+int wici_conv_forward(void *cuda_stream, const wici_conv_shape *s, const void *x, const void *w, float *y,
+                      void *workspace);
+
+/* dx = the gradient of sum(y * dy) with respect to x. */
+int wici_conv_backward_data(void *cuda_stream, const wici_conv_shape *s, const void *dy, const void *w, float *dx,
+                            void *workspace);
+
+/* dw = the gradient of sum(y * dy) with respect to w. */
+int wici_conv_backward_filter(void *cuda_stream, const wici_conv_shape *s, const void *x, const void *dy, float *dw,
+                              void *workspace);
+
+/* Synchronises cuda_stream and reports whether a bounded device wait of an
+ * earlier convolution call on `workspace` gave up (WICI_E_TIMEOUT; the word is
+ * then cleared) or not (WICI_OK). */
+int wici_conv_status(void *cuda_stream, void *workspace);
+
 /* Destroy the context (frees only what the library allocated).  (Sec. 5.4,
  * multiple clients: a client that disconnects releases its server thread.) */
 void wici_destroy(wici_ctx *ctx);

@@ -4,11 +4,16 @@
 // head g: the rows pack TPT tokens x `group` query heads (row r = token r/group,
 // head g*group + r%group), so each K/V tile serves the whole group.  Keys come
 // from the paged cache in blocks of 64 (four 16-key pages, fetched by 5-D TMA
-// through the page table).  Per block:
-//   S  = (Q_0 + Q_1) K^T          tcgen05.mma, M=128 rows, N=64 keys, fp32 in TMEM
-//   softmax (one row per thread, read from TMEM): online max/sum, P = exp2(s - m)
-//   O_blk = (P_0 + P_1) V         tcgen05.mma, N=d, V read as an MN-major operand
-//   O = O * corr + O_blk          in registers
+// through the page table).  Per block j:
+//   S_j  = (Q_0 + Q_1) K_j^T      tcgen05.mma, M=128 rows, N=64 keys, fp32 in TMEM
+//   softmax (one row per thread, read from TMEM): online max/sum, P_j = exp2(s - m_j)
+//   O_j  = (P_0 + P_1) V_j        tcgen05.mma, N=d, V read as an MN-major operand
+//   O = O * exp2(m_{j-1} - m_j) + O_j   in registers
+// S, P and O_j are double-buffered (two TMEM accumulators each for S and O_j, two
+// P tiles in shared memory), so the tensor cores work ahead of the softmax: the
+// MMA warp issues S_{j+2} as soon as the softmax has consumed S_j, and P_j V_j
+// runs while the softmax computes P_{j+1}; the softmax folds O_j into its
+// registers one block late.
 // Q and P are carried as two bf16 terms (hi + lo: 16 significant bits), K and V
 // are exact bf16: the products only meet bf16 K and V, whose own rounding is 2^-9,
 // and the two-term tiles leave room for a three-stage K/V ring (the kernel is
@@ -30,7 +35,7 @@ constexpr int AT_KEYS = 64;            // keys per block
 constexpr int AT_STAGES = 3;           // K/V ring depth
 constexpr int AT_TERMS = 2;            // bf16 terms of the Q and P operands
 constexpr int AT_THREADS = 192;
-constexpr uint32_t AT_TMEM_COLS = 256; // S: [0, 64), O block: [128, 128 + d)
+constexpr uint32_t AT_TMEM_COLS = 512; // S: [0, 64) and [64, 128); O blocks: [128, 128 + d) and [256, 256 + d)
 
 enum : int { SITE_AT_Q = 41, SITE_AT_KVE = 42, SITE_AT_KVF = 43, SITE_AT_S = 44, SITE_AT_P = 45, SITE_AT_O = 46,
              SITE_AT_DRAIN = 47 };
@@ -43,8 +48,8 @@ struct AttnSmem {
     static constexpr uint32_t P_BYTES = AT_ROWS * AT_KEYS * 2;           // one term
     static constexpr uint32_t OFF_Q = 0;                                 // [term]
     static constexpr uint32_t OFF_KV = AT_TERMS * Q_BYTES;               // [stage][K | V]
-    static constexpr uint32_t OFF_P = OFF_KV + AT_STAGES * 2 * KV_BYTES; // [term]
-    static constexpr uint32_t TOTAL = OFF_P + AT_TERMS * P_BYTES;
+    static constexpr uint32_t OFF_P = OFF_KV + AT_STAGES * 2 * KV_BYTES; // [buffer][term]
+    static constexpr uint32_t TOTAL = OFF_P + 2 * AT_TERMS * P_BYTES;
 };
 
 // K-major, 128-byte swizzle, 8-row groups 1024 B apart (Q, K and P operands)
@@ -108,7 +113,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                    const AttnArgs a) {
     using L = AttnSmem<D>;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t q_full, kv_full[AT_STAGES], kv_empty[AT_STAGES], s_full, p_full, o_full;
+    __shared__ __align__(8) uint64_t q_full, kv_full[AT_STAGES], kv_empty[AT_STAGES], s_full[2], p_full[2], o_full[2];
     __shared__ uint32_t s_tmem;
     __shared__ int s_issued;
 
@@ -128,9 +133,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             mbar_init(smem_u32(&kv_full[s]), 1);
             mbar_init(smem_u32(&kv_empty[s]), 1);
         }
-        mbar_init(smem_u32(&s_full), 1);
-        mbar_init(smem_u32(&p_full), 4);
-        mbar_init(smem_u32(&o_full), 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&s_full[b]), 1);
+            mbar_init(smem_u32(&p_full[b]), 4);
+            mbar_init(smem_u32(&o_full[b]), 1);
+        }
         fence_barrier_init();
         s_issued = 0;
     }
@@ -144,6 +151,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = s_tmem;
+    // buffer b of S at tmem + 64 b, of the O block at tmem + 128 + 128 b
     const uint32_t tm_s = tmem, tm_o = tmem + 128;
 
     if (warp == 0) {
@@ -189,6 +197,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                 if (!ok) return;
                 tc_fence_after();
                 const uint32_t kb = base + L::OFF_KV + (uint32_t)s * 2 * L::KV_BYTES;
+                const uint32_t sacc = tm_s + 64u * (uint32_t)(j & 1);
 #pragma unroll
                 for (int k = 0; k < D / 16; ++k) {
                     const uint32_t off = (uint32_t)(k / 4) * (AT_ROWS * 128) + 32u * (k % 4);
@@ -196,28 +205,32 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                     const uint64_t bd = at_desc_k(kb + koff);
 #pragma unroll
                     for (int t = 0; t < AT_TERMS; ++t)
-                        tc_mma(tm_s, at_desc_k(base + L::OFF_Q + t * L::Q_BYTES + off), bd, idesc_s, (k | t) != 0);
+                        tc_mma(sacc, at_desc_k(base + L::OFF_Q + t * L::Q_BYTES + off), bd, idesc_s, (k | t) != 0);
                 }
-                tc_commit(smem_u32(&s_full));
+                tc_commit(smem_u32(&s_full[j & 1]));
             };
             if (nb > 0) issue_s(0);
+            if (nb > 1) issue_s(1);
             for (int j = 0; j < nb && ok; ++j) {
-                const int s = j % AT_STAGES;
-                ok = mbar_wait(smem_u32(&p_full), j & 1, a.err, SITE_AT_P);   // P_j written, S_j read
+                const int s = j % AT_STAGES, b = j & 1;
+                // P_j written (and S_j read, and O_{j-2} folded) by the softmax
+                ok = mbar_wait(smem_u32(&p_full[b]), (j >> 1) & 1, a.err, SITE_AT_P);
                 if (!ok) break;
                 tc_fence_after();
                 const uint32_t vb = base + L::OFF_KV + (uint32_t)s * 2 * L::KV_BYTES + L::KV_BYTES;
+                const uint32_t pb = base + L::OFF_P + (uint32_t)b * AT_TERMS * L::P_BYTES;
 #pragma unroll
                 for (int k = 0; k < AT_KEYS / 16; ++k) {
                     // 16 keys = two 8-key groups of V rows; P columns 16k..16k+15
                     const uint64_t vd = at_desc_mn(vb + 2048u * k, AT_KEYS * 128);
 #pragma unroll
                     for (int t = 0; t < AT_TERMS; ++t)
-                        tc_mma(tm_o, at_desc_k(base + L::OFF_P + t * L::P_BYTES + 32u * k), vd, idesc_o, (k | t) != 0);
+                        tc_mma(tm_o + 128u * (uint32_t)b, at_desc_k(pb + t * L::P_BYTES + 32u * k), vd, idesc_o,
+                               (k | t) != 0);
                 }
-                tc_commit(smem_u32(&o_full));
+                tc_commit(smem_u32(&o_full[b]));
                 tc_commit(smem_u32(&kv_empty[s]));
-                if (j + 1 < nb) issue_s(j + 1);
+                if (j + 2 < nb) issue_s(j + 2);   // S buffer b was read before P_j was posted
             }
         }
     } else {  // ------------------------------------------------------- softmax / output
@@ -231,15 +244,29 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         float o[D];
 #pragma unroll
         for (int i = 0; i < D; ++i) o[i] = 0.f;
-        float m = -INFINITY, l = 0.f;
+        float m = -INFINITY, l = 0.f, corr_prev = 1.f;
         bool ok = true;
-        uint8_t *pbase = smem_raw + (base - smem_u32(smem_raw)) + L::OFF_P;
+        uint8_t *pbase0 = smem_raw + (base - smem_u32(smem_raw)) + L::OFF_P;
+        // O += the P.V block b of the previous iteration, in the new max's scale
+        auto fold = [&](int jb, float corr) {
+            const int b = jb & 1;
+            ok = ok && mbar_wait(smem_u32(&o_full[b]), (jb >> 1) & 1, a.err, SITE_AT_O);
+            tc_fence_after();
+#pragma unroll
+            for (int c0 = 0; c0 < D; c0 += 32) {
+                float ov[32];
+                tc_ld32(tm_o + 128u * (uint32_t)b + lane_base + c0, ov);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) o[c0 + i] = fmaf(o[c0 + i], corr, ov[i]);
+            }
+        };
         for (int j = 0; j < nb && ok; ++j) {
-            ok = mbar_wait(smem_u32(&s_full), j & 1, a.err, SITE_AT_S);
+            ok = mbar_wait(smem_u32(&s_full[j & 1]), (j >> 1) & 1, a.err, SITE_AT_S);
             tc_fence_after();
             float sv[AT_KEYS];
-            tc_ld32(tm_s + lane_base, sv);
-            tc_ld32(tm_s + lane_base + 32, sv + 32);
+            tc_ld32(tm_s + 64u * (uint32_t)(j & 1) + lane_base, sv);
+            tc_ld32(tm_s + 64u * (uint32_t)(j & 1) + lane_base + 32, sv + 32);
+            uint8_t *pbase = pbase0 + (size_t)(j & 1) * AT_TERMS * L::P_BYTES;
             float bm = -INFINITY;
 #pragma unroll
             for (int c = 0; c < AT_KEYS; ++c) {
@@ -275,17 +302,14 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             fence_proxy_async_smem();   // generic-proxy writes of P before the MMA reads them
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&p_full));
-            ok = ok && mbar_wait(smem_u32(&o_full), j & 1, a.err, SITE_AT_O);
-            tc_fence_after();
-#pragma unroll
-            for (int c0 = 0; c0 < D; c0 += 32) {
-                float ov[32];
-                tc_ld32(tm_o + lane_base + c0, ov);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) o[c0 + i] = fmaf(o[c0 + i], corr, ov[i]);
-            }
+            if (lane == 0) mbar_arrive(smem_u32(&p_full[j & 1]));
+            // fold the previous block, whose P.V ran while this block's P was computed;
+            // this also frees its P tile and O accumulator for block j + 1
+            if (j > 0) fold(j - 1, corr_prev);
+            tc_fence_before();
+            corr_prev = corr;
         }
+        if (ok && nb > 0) fold(nb - 1, corr_prev);
         if (ok && row_ok && tok < a.T) {
             const float inv = 1.0f / l;
             const size_t off = (size_t)tok * a.nq * D + (size_t)head * D;

@@ -134,6 +134,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                    const __grid_constant__ CUtensorMap map_w1, const __grid_constant__ CUtensorMap map_w2, int T,
                    int N, int K, int *err, const Epi epi) {
     static_assert(WT == 1 || WT == kTerms, "one exact bf16 weight term, or three");
+    // activation terms multiplied against a bf16 weight: the epilogue type states it
+    constexpr int AT = Epi::kATerms;
+    static_assert(AT >= 1 && AT <= kTerms, "activation terms");
     using G = TcTile<BN>;
     constexpr int S = G::STAGES;
     extern __shared__ uint8_t smem_raw[];
@@ -186,10 +189,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     const uint32_t st = base + (uint32_t)s * G::STAGE_BYTES;
                     const uint32_t fb = smem_u32(&full_bar[s]);
                     // term j meets the activation terms i <= 2 - j only
-                    mbar_arrive_expect_tx(fb, (uint32_t)(kTerms - j) * TC_A_BYTES + G::B_BYTES);
+                    const int na = WT == 1 ? AT : kTerms - j;
+                    mbar_arrive_expect_tx(fb, (uint32_t)na * TC_A_BYTES + G::B_BYTES);
                     tma_load_2d(st, &map_a0, kb * TC_BK, m0, fb);
-                    if (j < 2) tma_load_2d(st + TC_A_BYTES, &map_a1, kb * TC_BK, m0, fb);
-                    if (j < 1) tma_load_2d(st + 2 * TC_A_BYTES, &map_a2, kb * TC_BK, m0, fb);
+                    if (na > 1) tma_load_2d(st + TC_A_BYTES, &map_a1, kb * TC_BK, m0, fb);
+                    if (na > 2) tma_load_2d(st + 2 * TC_A_BYTES, &map_a2, kb * TC_BK, m0, fb);
                     tma_load_2d(st + kTerms * TC_A_BYTES, j == 0 ? &map_w : j == 1 ? &map_w1 : &map_w2, kb * TC_BK, n0,
                                 fb);
                     s_issued = it + 1;
@@ -215,7 +219,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         ok = mbar_wait(smem_u32(&full_bar[s]), (it / S) & 1, err, SITE_TC_FULL);
                         if (!ok) break;
                         tc_fence_after();
-                        const int nt = WT == 1 ? kTerms : kTerms - kk / nk;   // activation terms meeting this weight term
+                        const int nt = WT == 1 ? AT : kTerms - kk / nk;   // activation terms meeting this weight term
                         const uint32_t st = base + (uint32_t)s * G::STAGE_BYTES;
                         // descriptors of k-step 0; each k-step of 16 elements is 32 bytes further
                         const uint64_t bd0 = tc_desc_sw128(st + kTerms * TC_A_BYTES);

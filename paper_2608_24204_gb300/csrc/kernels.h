@@ -54,6 +54,11 @@ struct PrefillMaps {
 };
 
 
+// A bf16 tensor map with 128-byte swizzle: dims / box / element strides innermost
+// first, strides_bytes[i] the byte stride of dimension i + 1 (false on failure).
+bool encode_tiled(CUtensorMap *m, int rank, const void *ptr, const uint64_t *dims, const uint64_t *strides_bytes,
+                  const uint32_t *box, const uint32_t *elem_strides);
+
 // Encodes every tensor map of `m`; returns an error message or nullptr.
 const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m);
 

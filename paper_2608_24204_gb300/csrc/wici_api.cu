@@ -30,6 +30,8 @@ struct wici_ctx {
     std::vector<char> loaded;        // per canonical tensor
     int n_required = 0, n_loaded = 0;
     cudaGraphExec_t step_exec = nullptr;
+    cudaEvent_t step_done[2] = {nullptr, nullptr};  // SM-share contexts: after every decode step
+    long long steps_launched = 0;
     PrefillMaps maps;
     int32_t *pinned = nullptr;       // host staging: [0] token in, [1] token out, [2] err
     std::string err;
@@ -328,6 +330,10 @@ int wici_create(const wici_config *cfg, void *cuda_stream, void *weight_dev, voi
     do {
         if ((e = setup_kernels()) != cudaSuccess) break;
         if ((e = cudaHostAlloc((void **)&c->pinned, 64, cudaHostAllocDefault)) != cudaSuccess) break;
+        if (p.cfg.max_sms > 0 &&
+            ((e = cudaEventCreateWithFlags(&c->step_done[0], cudaEventDisableTiming)) != cudaSuccess ||
+             (e = cudaEventCreateWithFlags(&c->step_done[1], cudaEventDisableTiming)) != cudaSuccess))
+            break;
         if ((e = cudaMemsetAsync(c->bufs.ctrl, 0, CTRL_WORDS * sizeof(int), c->stream)) != cudaSuccess) break;
         // cache slots past the length are read (and weighted by zero) by the
         // tensor-core attention: they must hold finite values from the start
@@ -603,10 +609,31 @@ static int begin_decode(wici_ctx *c, int32_t n_steps, int32_t token_in) {
     return WICI_OK;
 }
 
+// One decode step on the stream: the captured graph, or, for a context on an SM
+// share, the step kernel launched directly (graph replays of different contexts
+// were measured to run one after the other, while direct launches of the
+// persistent step kernel on disjoint SM shares run at the same time).
+// At most this many decode steps of an SM-share context are queued at once:
+// with deep queues the steps of two tenants were measured to alternate on the
+// GPU instead of overlapping.
+constexpr int kShareDepth = 2;
+
+static cudaError_t launch_step(wici_ctx *c) {
+    if (c->plan.cfg.max_sms > 0 && decode_is_persistent(c->plan)) {
+        cudaEvent_t ev = c->step_done[c->steps_launched % kShareDepth];
+        cudaError_t e = c->steps_launched >= kShareDepth ? cudaEventSynchronize(ev) : cudaSuccess;
+        if (e == cudaSuccess) e = enqueue_decode_step(c->plan, c->bufs, c->stream, false, nullptr);
+        if (e == cudaSuccess) e = cudaEventRecord(ev, c->stream);
+        if (e == cudaSuccess) ++c->steps_launched;
+        return e;
+    }
+    return cudaGraphLaunch(c->step_exec, c->stream);
+}
+
 int wici_decode_step(wici_ctx *c, int32_t token_in, float *logits_out, int32_t *token_out) {
     if (!c) return fail(nullptr, WICI_E_ARG, "null context");
     if (int rc = begin_decode(c, 1, token_in)) return rc;
-    CUDA_TRY(c, cudaGraphLaunch(c->step_exec, c->stream));
+    CUDA_TRY(c, launch_step(c));
     if (logits_out)
         CUDA_TRY(c, cudaMemcpyAsync(logits_out, c->bufs.logits, (size_t)c->plan.V * 4, cudaMemcpyDeviceToHost,
                                     c->stream));
@@ -617,7 +644,7 @@ int wici_decode(wici_ctx *c, int32_t n_steps, int32_t token_in, int32_t *tokens_
     if (!c) return fail(nullptr, WICI_E_ARG, "null context");
     if (n_steps < 1) return fail(c, WICI_E_ARG, "n_steps must be >= 1");
     if (int rc = begin_decode(c, n_steps, token_in)) return rc;
-    for (int i = 0; i < n_steps; ++i) CUDA_TRY(c, cudaGraphLaunch(c->step_exec, c->stream));
+    for (int i = 0; i < n_steps; ++i) CUDA_TRY(c, launch_step(c));
     if (tokens_out)
         CUDA_TRY(c, cudaMemcpyAsync(tokens_out, c->bufs.hist + c->kv_len + 1, (size_t)n_steps * 4,
                                     cudaMemcpyDeviceToHost, c->stream));
@@ -741,6 +768,8 @@ void wici_destroy(wici_ctx *c) {
     if (!c) return;
     if (c->stream) cudaStreamSynchronize(c->stream);
     if (c->step_exec) cudaGraphExecDestroy(c->step_exec);
+    for (cudaEvent_t e : c->step_done)
+        if (e) cudaEventDestroy(e);
     if (c->pinned) cudaFreeHost(c->pinned);
     delete c;
 }

@@ -23,7 +23,9 @@ STATUS_NAMES = {0: "WICI_OK", -1: "WICI_E_ARG", -2: "WICI_E_STATE", -3: "WICI_E_
 EXPORTS = ("wici_get_sizes", "wici_create", "wici_load_weights", "wici_load_weights_q8", "wici_prefill",
            "wici_decode_step",
            "wici_decode", "wici_reset", "wici_set_page_table", "wici_kv_len", "wici_last_error",
-           "wici_profile_decode", "wici_check_bounded_wait", "wici_destroy", "wici_lm_head_argmax_noalloc")
+           "wici_profile_decode", "wici_check_bounded_wait", "wici_destroy", "wici_lm_head_argmax_noalloc",
+           "wici_conv_workspace_bytes", "wici_conv_forward", "wici_conv_backward_data", "wici_conv_backward_filter",
+           "wici_conv_status")
 
 
 class wici_config(ctypes.Structure):
@@ -82,10 +84,18 @@ def lib():
         L.wici_destroy.argtypes = [vp]
         L.wici_destroy.restype = None
         L.wici_lm_head_argmax_noalloc.argtypes = [vp, vp, vp, vp, i32, i32, ctypes.c_float, vp, vp]
+        cs = P(wici_conv_shape)
+        L.wici_conv_workspace_bytes.argtypes = [cs, P(ctypes.c_size_t)]
+        L.wici_conv_forward.argtypes = [vp, cs, vp, vp, vp, vp]
+        L.wici_conv_backward_data.argtypes = [vp, cs, vp, vp, vp, vp]
+        L.wici_conv_backward_filter.argtypes = [vp, cs, vp, vp, vp, vp]
+        L.wici_conv_status.argtypes = [vp, vp]
         for name in ("wici_get_sizes", "wici_create", "wici_load_weights", "wici_load_weights_q8", "wici_prefill",
                      "wici_decode_step",
                      "wici_decode", "wici_reset", "wici_set_page_table", "wici_profile_decode",
-                     "wici_check_bounded_wait", "wici_lm_head_argmax_noalloc"):
+                     "wici_check_bounded_wait", "wici_lm_head_argmax_noalloc", "wici_conv_workspace_bytes",
+                     "wici_conv_forward", "wici_conv_backward_data", "wici_conv_backward_filter",
+                     "wici_conv_status"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -219,6 +229,34 @@ def wici_lm_head_argmax_noalloc(stream: int, lm_head_dev: int, norm_gain_dev: in
     scratch is a fixed array inside the library.  Enqueued on `stream`."""
     _check(lib().wici_lm_head_argmax_noalloc(stream, lm_head_dev, norm_gain_dev, x_dev, hidden, vocab, rms_eps,
                                               logits_dev, token_dev))
+
+
+# ------------------------------------------------------- CNN-training sample
+class wici_conv_shape(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int32), ("c", ctypes.c_int32), ("h", ctypes.c_int32), ("w", ctypes.c_int32),
+                ("k", ctypes.c_int32)]
+
+
+def wici_conv_workspace_bytes(shape: wici_conv_shape) -> int:
+    out = ctypes.c_size_t()
+    _check(lib().wici_conv_workspace_bytes(ctypes.byref(shape), ctypes.byref(out)))
+    return int(out.value)
+
+
+def wici_conv_forward(stream: int, shape: wici_conv_shape, x: int, w: int, y: int, ws: int) -> None:
+    _check(lib().wici_conv_forward(stream, ctypes.byref(shape), x, w, y, ws))
+
+
+def wici_conv_backward_data(stream: int, shape: wici_conv_shape, dy: int, w: int, dx: int, ws: int) -> None:
+    _check(lib().wici_conv_backward_data(stream, ctypes.byref(shape), dy, w, dx, ws))
+
+
+def wici_conv_backward_filter(stream: int, shape: wici_conv_shape, x: int, dy: int, dw: int, ws: int) -> None:
+    _check(lib().wici_conv_backward_filter(stream, ctypes.byref(shape), x, dy, dw, ws))
+
+
+def wici_conv_status(stream: int, ws: int) -> None:
+    _check(lib().wici_conv_status(stream, ws))
 
 
 # ------------------------------------------------------------- convenience

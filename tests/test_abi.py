@@ -26,7 +26,7 @@ def declared_entry_points():
 
 def test_library_exports_every_declared_entry_point():
     names = declared_entry_points()
-    assert len(names) == 15
+    assert len(names) == 20
     L = wici.lib()
     for n in names:
         assert hasattr(L, n), n
@@ -58,6 +58,15 @@ def test_q8_sizes_hold_codes_and_block_scales():
     assert abs((b.weight_bytes - q.weight_bytes) - saved) < 1_000_000
     assert q.workspace_bytes - b.workspace_bytes >= 3 * 2 * (2 * cfg.ffn_dim * cfg.hidden)
     assert q.kv_bytes == b.kv_bytes
+
+
+def test_conv_shape_checks_and_workspace_size():
+    s = wici.wici_conv_shape(4, 1024, 224, 224, 1024)
+    assert wici.wici_conv_workspace_bytes(s) == 256 + 9 * 1024 * 1024 * 2
+    for bad in ((4, 1000, 224, 224, 1024), (4, 1024, 223, 224, 1024), (0, 256, 8, 8, 256)):
+        with pytest.raises(wici.WiciError) as e:
+            wici.wici_conv_workspace_bytes(wici.wici_conv_shape(*bad))
+        assert e.value.status == wici.WICI_E_ARG
 
 
 def test_q8_rejects_widths_that_are_not_multiples_of_256():
