@@ -195,14 +195,14 @@ def cpu_oracle_sample(weights, budget_s: float = 20.0):
                       f"(numpy fp64, {dt:.1f} s)"}
 
 
-def measure_agentic(weights, WiciModel, torch, pk, runs: int = 3):
+def measure_agentic(weights, WiciModel, torch, pk, runs: int = 3, cfg=None):
     """The agentic long-context workload at the 8B shape: 4 turns, each a
     2048-token chunk appended to the same cache (prefill) and then 64 greedy
     decode steps, ending at 8448 cached tokens.  Reported: the four chunk
     prefills in aggregate (the 8K-token prefill) against the bf16 tensor peak,
     and the decode steps against the HBM peak.  CUDA events on the library's
     stream; one untimed run first, then the median of `runs`."""
-    cfg = gen.LLAMA_8B_AGENTIC
+    cfg = cfg or gen.LLAMA_8B_AGENTIC
     T, steps, turns = cfg.prompt_len, cfg.decode_steps, cfg.turns
     model = WiciModel(cfg, max_tokens=turns * (T + steps), max_chunk=T).load(weights)
     prompts = [gen.make_prompt(cfg, T, seed=s) for s in cfg.prompt_seeds]
@@ -443,6 +443,18 @@ def run_ours(args):
     dev = torch.cuda.current_device()
     pk = peaks()
 
+    if QUICK and args.workload != "request":
+        # profiling runs of the other measured workloads, at CFG's depth
+        if args.workload == "agentic":
+            cfg = gen.LLAMA_8B_AGENTIC.with_(n_layers=CFG.n_layers)
+            out = measure_agentic(gen.make_weights(cfg), WiciModel, torch, pk, runs=args.steps, cfg=cfg)
+        elif args.workload == "q8":
+            out = measure_q8(gen.make_weights(CFG), WiciModel, torch, pk, runs=args.steps)
+        else:
+            out = measure_cnn_train(torch, pk, runs=args.steps)
+        print(json.dumps({"profile_run": True, "workload": args.workload, **out}), flush=True)
+        return 0
+
     t_setup = time.time()
     weights = gen.make_weights(CFG)
     max_tokens = PROMPT + DECODE + 16
@@ -617,6 +629,8 @@ def main():
     ap.add_argument("--quick", action="store_true", help="profiling run: timed requests only")
     ap.add_argument("--decode-steps", type=int, default=0, help="profiling run: decode steps per request")
     ap.add_argument("--layers", type=int, default=0, help="profiling run: fewer layers (small ncu case)")
+    ap.add_argument("--workload", default="request", choices=["request", "agentic", "q8", "cnn"],
+                    help="profiling run (--quick): which measured workload to run")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)
