@@ -17,9 +17,11 @@
 //
 // Weights in the 8-bit block format arrive dequantised as WT = 3 bf16 terms
 // W = W_0 + W_1 + W_2 (exact: a code times an fp16 scale has at most 18
-// significant bits).  The K loop then runs once per weight term j, issuing the
-// products A_i W_j with i + j <= 2 (the others lie below 2^-24 of the result):
-// 3 + 2 + 1 MMAs per k-step instead of 3.
+// significant bits).  The K loop then runs once per weight term j < AT, issuing
+// the products A_i W_j with i + j < AT, AT the activation terms of the GEMM:
+// with AT = 3 that is 3 + 2 + 1 MMAs per k-step (the dropped products lie below
+// 2^-24 of the result); with AT = 2 it is 2 + 1, the weight then carried at the
+// activations' own 16 significant bits.
 //
 // Persistent: one CTA per SM walks the output tiles (M tiles fastest, so the
 // CTAs that run together share a weight tile through L2) with three warp roles:
@@ -148,7 +150,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     const int ntm = (T + TC_BM - 1) / TC_BM, ntn = (N + BN - 1) / BN;
     const int ntiles = ntm * ntn;
     const int nk = (K + TC_BK - 1) / TC_BK;
-    const int nkk = nk * WT;                      // k-blocks of all weight terms
+    constexpr int WU = WT == 1 ? 1 : Epi::kATerms;  // weight terms used
+    const int nkk = nk * WU;                      // k-blocks of all weight terms
     const int ngroups = (nkk + TC_GROUP - 1) / TC_GROUP;
     const uint32_t base = (smem_u32(smem_raw) + 1023u) & ~1023u;
 
@@ -189,7 +192,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     const uint32_t st = base + (uint32_t)s * G::STAGE_BYTES;
                     const uint32_t fb = smem_u32(&full_bar[s]);
                     // term j meets the activation terms i <= 2 - j only
-                    const int na = WT == 1 ? AT : kTerms - j;
+                    const int na = AT - j;
                     mbar_arrive_expect_tx(fb, (uint32_t)na * TC_A_BYTES + G::B_BYTES);
                     tma_load_2d(st, &map_a0, kb * TC_BK, m0, fb);
                     if (na > 1) tma_load_2d(st + TC_A_BYTES, &map_a1, kb * TC_BK, m0, fb);
@@ -219,7 +222,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         ok = mbar_wait(smem_u32(&full_bar[s]), (it / S) & 1, err, SITE_TC_FULL);
                         if (!ok) break;
                         tc_fence_after();
-                        const int nt = WT == 1 ? AT : kTerms - kk / nk;   // activation terms meeting this weight term
+                        const int nt = WT == 1 ? AT : AT - kk / nk;   // activation terms meeting this weight term
                         const uint32_t st = base + (uint32_t)s * G::STAGE_BYTES;
                         // descriptors of k-step 0; each k-step of 16 elements is 32 bytes further
                         const uint64_t bd0 = tc_desc_sw128(st + kTerms * TC_A_BYTES);

@@ -323,7 +323,7 @@ __global__ void qk_norm_rope_kernel(const float *raw, const uint16_t *qn, const 
 // row-major [rows][K] matrix.  The product is exact in fp32 (at most 18
 // significant bits), and so is its split into three terms.  8 elements per
 // thread: one 8-byte code load, one scale, one 16-byte store per term.
-__global__ void q8_dequant_terms_kernel(const uint8_t *src, int rows, int K, const Terms out) {
+__global__ void q8_dequant_terms_kernel(const uint8_t *src, int rows, int K, const Terms out, int nterms) {
     const int per_row = K / 8;
     const size_t rb = (size_t)K + (size_t)K / 16;
     const long long n = (long long)rows * per_row;
@@ -348,17 +348,17 @@ __global__ void q8_dequant_terms_kernel(const uint8_t *src, int rows, int K, con
         const size_t o = (size_t)r * K + (size_t)c * 8;
 #pragma unroll
         for (int q = 0; q < kTerms; ++q)
-            *reinterpret_cast<uint4 *>(out.p[q] + o) = make_uint4(t[q][0], t[q][1], t[q][2], t[q][3]);
+            if (q < nterms) *reinterpret_cast<uint4 *>(out.p[q] + o) = make_uint4(t[q][0], t[q][1], t[q][2], t[q][3]);
     }
 }
 
-static cudaError_t dequant_terms(const Plan &p, const Bufs &b, const uint16_t *W, int rows, int K, cudaStream_t st,
-                                 LaunchHook *hook) {
+static cudaError_t dequant_terms(const Plan &p, const Bufs &b, const uint16_t *W, int rows, int K, int nterms,
+                                 cudaStream_t st, LaunchHook *hook) {
     const long long n = (long long)rows * (K / 8);
     const int grid = (int)((n + 255) / 256 < 8 * p.num_sms ? (n + 255) / 256 : 8 * p.num_sms);
     if (hook) hook->before("prefill_q8_dequant");
     q8_dequant_terms_kernel<<<grid, 256, 0, st>>>(reinterpret_cast<const uint8_t *>(W), rows, K,
-                                                 Terms{{b.Wt[0], b.Wt[1], b.Wt[2]}});
+                                                 Terms{{b.Wt[0], b.Wt[1], b.Wt[2]}}, nterms);
     if (hook) hook->after("prefill_q8_dequant");
     return cudaGetLastError();
 }
@@ -574,6 +574,7 @@ static cudaError_t gemm(const Plan &p, int bn, const CUtensorMap *a, const WOper
 
 // bf16: the layer's own matrix; 8-bit format: dequantise the layer's rows into
 // the workspace terms first (stream order makes the previous GEMM finish reading them)
+template <class Epi>
 static cudaError_t weight_operand(const Plan &p, const Bufs &b, const CUtensorMap &bf16_map,
                                   const CUtensorMap *terms, const uint16_t *rows, int n_rows, int K, cudaStream_t st,
                                   LaunchHook *hook, WOperand *w) {
@@ -582,7 +583,7 @@ static cudaError_t weight_operand(const Plan &p, const Bufs &b, const CUtensorMa
         return cudaSuccess;
     }
     *w = WOperand{{&terms[0], &terms[1], &terms[2]}, kTerms};
-    return dequant_terms(p, b, rows, n_rows, K, st, hook);
+    return dequant_terms(p, b, rows, n_rows, K, Epi::kATerms, st, hook);   // the weight terms the GEMM uses
 }
 
 cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMaps &mp, cudaStream_t st, int P,
@@ -600,7 +601,7 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         PEpiQKV eq = {{{b.Q[0], b.Q[1], b.Q[2]}}, kvl, b.pages, b.rope, p.cfg.qkv_bias ? b.W + lo.bqkv : nullptr, P, p.qdim,
                       p.kvdim, p.d, p.nkv, p.kv_page_elems, p.qk_norm ? b.QKraw : nullptr};
         WOperand w;
-        if ((e = weight_operand(p, b, p.q8 ? mp.wt_qkv[0] : mp.wqkv[l], mp.wt_qkv, b.W + lo.wqkv, p.nqkv, p.H, st,
+        if ((e = weight_operand<PEpiQKV>(p, b, p.q8 ? mp.wt_qkv[0] : mp.wqkv[l], mp.wt_qkv, b.W + lo.wqkv, p.nqkv, p.H, st,
                                 hook, &w)) != cudaSuccess)
             return e;
         if ((e = gemm(p, mp.bn_qkv, mp.a, w, T, p.nqkv, p.H, err, eq, st, hook, "prefill_qkv")) != cudaSuccess)
@@ -625,7 +626,7 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         if (hook) hook->after("prefill_attention");
         if (e != cudaSuccess) return e;
         // A6: O projection + residual
-        if ((e = weight_operand(p, b, p.q8 ? mp.wt_o[0] : mp.wo[l], mp.wt_o, b.W + lo.wo, p.H, p.qdim, st, hook,
+        if ((e = weight_operand<PEpiResidual>(p, b, p.q8 ? mp.wt_o[0] : mp.wo[l], mp.wt_o, b.W + lo.wo, p.H, p.qdim, st, hook,
                                 &w)) != cudaSuccess)
             return e;
         if ((e = gemm(p, mp.bn_o, mp.o, w, T, p.H, p.qdim, err, PEpiResidual{b.X, p.H}, st, hook,
@@ -634,14 +635,14 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         // A7: RMSNorm + gate/up + SwiGLU
         rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.ffn_norm, A, p.H, p.cfg.rms_eps);
         const Terms M = {{b.M[0], b.M[1], b.M[2]}};
-        if ((e = weight_operand(p, b, p.q8 ? mp.wt_gu[0] : mp.wgu[l], mp.wt_gu, b.W + lo.wgu, 2 * p.F, p.H, st,
+        if ((e = weight_operand<PEpiSwiGLU>(p, b, p.q8 ? mp.wt_gu[0] : mp.wgu[l], mp.wt_gu, b.W + lo.wgu, 2 * p.F, p.H, st,
                                 hook, &w)) != cudaSuccess)
             return e;
         if ((e = gemm(p, mp.bn_gu, mp.a, w, T, 2 * p.F, p.H, err, PEpiSwiGLU{M, p.F}, st, hook,
                       "prefill_gate_up")) != cudaSuccess)
             return e;
         // A8: down projection + residual
-        if ((e = weight_operand(p, b, p.q8 ? mp.wt_d[0] : mp.wd[l], mp.wt_d, b.W + lo.wd, p.H, p.F, st, hook,
+        if ((e = weight_operand<PEpiResidual>(p, b, p.q8 ? mp.wt_d[0] : mp.wd[l], mp.wt_d, b.W + lo.wd, p.H, p.F, st, hook,
                                 &w)) != cudaSuccess)
             return e;
         if ((e = gemm(p, mp.bn_d, mp.m, w, T, p.H, p.F, err, PEpiResidual{b.X, p.H}, st, hook,
