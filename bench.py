@@ -221,7 +221,18 @@ def measure_agentic(weights, WiciModel, torch, pk, runs: int = 3, cfg=None):
         if r > 0:
             pf_ms.append([e[0].elapsed_time(e[1]) for e in ev])
             dec_ms.append([e[1].elapsed_time(e[2]) for e in ev])
+    # the last turn's prefill kernels one by one (CUDA events around every launch)
+    from paper_2608_24204_gb300 import wici
+    model.reset()
+    for t in range(turns - 1):
+        model.prefill(prompts[t])
+        model.decode(steps)
+    prof = wici.wici_profile_prefill(model.ctx, prompts[turns - 1])
     model.close()
+    P4 = (turns - 1) * (T + steps)
+    attn_flops = cfg.n_layers * cfg.n_q_heads * cfg.head_dim * 4 * (T * P4 + T * (T + 1) // 2)
+    n_a, ms_a = prof.get("prefill_attention", (0, float("nan")))
+    attn_tf = attn_flops / (ms_a / 1000.0) / 1e12
     i = sorted(range(runs), key=lambda k: sum(pf_ms[k]))[runs // 2]
     pf, dec = pf_ms[i], dec_ms[i]
     flops = [gen.prefill_flops(cfg, T, t * (T + steps)) for t in range(turns)]
@@ -235,6 +246,10 @@ def measure_agentic(weights, WiciModel, torch, pk, runs: int = 3, cfg=None):
             "prefill_roofline": {"bound": "tensor", "achieved": tf, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
                                  "frac": tf / pk["bf16_tflops"],
                                  "frac_of_sustained": tf / pk["bf16_tflops_sustained"]},
+            "last_turn_kernels_ms": {k: v[1] for k, v in prof.items()},
+            "last_turn_attention": {"bound": "tensor", "launches": n_a, "ms": ms_a, "achieved": attn_tf,
+                                    "peak": pk["bf16_tflops"], "unit": "TFLOP/s", "frac": attn_tf / pk["bf16_tflops"],
+                                    "flops": attn_flops, "cached_before": P4, "chunk": T},
             "decode_tok_s": turns * steps / dec_s, "decode_gbs": dec_bytes / dec_s / 1e9,
             "decode_frac_of_8tbs": dec_bytes / dec_s / 1e9 / NOMINAL_HBM_GBS,
             "decode_frac_of_measured_hbm": dec_bytes / dec_s / 1e9 / pk["hbm_gbs"],

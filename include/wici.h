@@ -199,6 +199,15 @@ const char *wici_last_error(const wici_ctx *ctx);
 int wici_profile_decode(wici_ctx *ctx, int32_t n_steps, const char **names, int32_t *launches,
                         double *total_ms, int32_t cap, int32_t *n_kinds);
 
+/* Measurement of the prefill's kernels (Sec. 5.1, TTFT), like wici_profile_decode:
+ * appends the n host tokens exactly as wici_prefill does (kv_len += n), with
+ * every launch bracketed by CUDA events on the context's stream.  For each
+ * kernel kind i < *n_kinds: names[i] ("prefill_qkv", "prefill_attention",
+ * "prefill_o_proj", "prefill_gate_up", "prefill_down", ...; static strings),
+ * launches[i] and total_ms[i].  Arrays have room for `cap` entries. */
+int wici_profile_prefill(wici_ctx *ctx, const int32_t *tokens, int32_t n, const char **names, int32_t *launches,
+                         double *total_ms, int32_t cap, int32_t *n_kinds);
+
 /* Failure detection (no paper counterpart).
  * Self-test of the bounded device wait: launches one CTA that waits on an
  * mbarrier nobody arrives at, giving up after `limit_ns` nanoseconds.  Returns

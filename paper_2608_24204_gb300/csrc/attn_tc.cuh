@@ -16,10 +16,12 @@
 // registers one block late.
 // Q and P are carried as two bf16 terms (hi + lo: 16 significant bits), K and V
 // are exact bf16: the products only meet bf16 K and V, whose own rounding is 2^-9,
-// and the two-term tiles leave room for a three-stage K/V ring (the kernel is
-// bound by the K/V bytes it keeps in flight).  Warp roles: 0 TMA producer,
-// 1 TMEM owner + MMA issuer, 2..5
-// softmax / output (TMEM lane quadrant = warp % 4).  Every wait is bounded.
+// and the two-term tiles leave room for a three-stage K/V ring.  Warp roles:
+// 0 TMA producer, 1 TMEM owner + MMA issuer, 2..9 softmax / output: two warps
+// per TMEM lane quadrant (warp % 4), one for keys 0..31 and output columns
+// [0, d/2) of its 32 rows, the other for keys 32..63 and columns [d/2, d); the
+// pair exchanges each block's row maxima through shared memory.  Every wait is
+// bounded.
 #pragma once
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -34,7 +36,7 @@ constexpr int AT_ROWS = 128;           // query rows per tile (TMEM lanes)
 constexpr int AT_KEYS = 64;            // keys per block
 constexpr int AT_STAGES = 3;           // K/V ring depth
 constexpr int AT_TERMS = 2;            // bf16 terms of the Q and P operands
-constexpr int AT_THREADS = 192;
+constexpr int AT_THREADS = 320;     // producer, MMA, 8 softmax warps (two per TMEM lane quadrant)
 constexpr uint32_t AT_TMEM_COLS = 512; // S: [0, 64) and [64, 128); O blocks: [128, 128 + d) and [256, 256 + d)
 
 enum : int { SITE_AT_Q = 41, SITE_AT_KVE = 42, SITE_AT_KVF = 43, SITE_AT_S = 44, SITE_AT_P = 45, SITE_AT_O = 46,
@@ -116,6 +118,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     __shared__ __align__(8) uint64_t q_full, kv_full[AT_STAGES], kv_empty[AT_STAGES], s_full[2], p_full[2], o_full[2];
     __shared__ uint32_t s_tmem;
     __shared__ int s_issued;
+    __shared__ float s_rowmax[2][AT_ROWS];      // [key half][row]: each block's row maxima, the row sums at the end
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int g = blockIdx.y;
@@ -135,7 +138,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&s_full[b]), 1);
-            mbar_init(smem_u32(&p_full[b]), 4);
+            mbar_init(smem_u32(&p_full[b]), 8);
             mbar_init(smem_u32(&o_full[b]), 1);
         }
         fence_barrier_init();
@@ -234,16 +237,19 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             }
         }
     } else {  // ------------------------------------------------------- softmax / output
+        constexpr int HK = AT_KEYS / 2, HD = D / 2;   // keys and output columns per warp of a pair
         const int qd = warp & 3;                   // TMEM lane quadrant
+        const int hc = (warp - 2) >> 2;            // which half of the keys and of the output columns
         const int r = qd * 32 + lane;              // tile row
         const bool row_ok = r < a.tpt * a.group;
         const int tok = t0 + r / a.group;          // chunk token of this row
         const int qpos = a.P + tok;                // its absolute position
         const int head = g * a.group + r % a.group;
         const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
-        float o[D];
+        const uint32_t pair_bar = 1 + qd;          // named barrier of the two warps of this quadrant
+        float o[HD];
 #pragma unroll
-        for (int i = 0; i < D; ++i) o[i] = 0.f;
+        for (int i = 0; i < HD; ++i) o[i] = 0.f;
         float m = -INFINITY, l = 0.f, corr_prev = 1.f;
         bool ok = true;
         uint8_t *pbase0 = smem_raw + (base - smem_u32(smem_raw)) + L::OFF_P;
@@ -253,27 +259,44 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             ok = ok && mbar_wait(smem_u32(&o_full[b]), (jb >> 1) & 1, a.err, SITE_AT_O);
             tc_fence_after();
 #pragma unroll
-            for (int c0 = 0; c0 < D; c0 += 32) {
+            for (int c0 = 0; c0 < HD; c0 += 32) {
                 float ov[32];
-                tc_ld32(tm_o + 128u * (uint32_t)b + lane_base + c0, ov);
+                tc_ld32(tm_o + 128u * (uint32_t)b + lane_base + hc * HD + c0, ov);
 #pragma unroll
                 for (int i = 0; i < 32; ++i) o[c0 + i] = fmaf(o[c0 + i], corr, ov[i]);
             }
         };
-        for (int j = 0; j < nb && ok; ++j) {
-            ok = mbar_wait(smem_u32(&s_full[j & 1]), (j >> 1) & 1, a.err, SITE_AT_S);
+        for (int j = 0; j < nb; ++j) {
+            ok = ok && mbar_wait(smem_u32(&s_full[j & 1]), (j >> 1) & 1, a.err, SITE_AT_S);
             tc_fence_after();
-            float sv[AT_KEYS];
-            tc_ld32(tm_s + 64u * (uint32_t)(j & 1) + lane_base, sv);
-            tc_ld32(tm_s + 64u * (uint32_t)(j & 1) + lane_base + 32, sv + 32);
+            float sv[HK];
+            tc_ld32(tm_s + 64u * (uint32_t)(j & 1) + lane_base + hc * HK, sv);
             uint8_t *pbase = pbase0 + (size_t)(j & 1) * AT_TERMS * L::P_BYTES;
             float bm = -INFINITY;
 #pragma unroll
-            for (int c = 0; c < AT_KEYS; ++c) {
-                const int key = j * AT_KEYS + c;
+            for (int c = 0; c < HK; ++c) {
+                const int key = j * AT_KEYS + hc * HK + c;
                 sv[c] = (row_ok && key <= qpos) ? sv[c] * a.scale_log2 : -INFINITY;
                 bm = fmaxf(bm, sv[c]);
             }
+            // the row's block maximum over both halves
+            s_rowmax[hc][r] = bm;
+            // the pair leaves the loop together: the barrier also ANDs the two warps'
+            // wait results, so a wait that gave up in one warp never strands the other
+            uint32_t both_ok;
+            asm volatile(
+                "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 q, %1, 0;\n\t"
+                "bar.red.and.pred p, %2, 64, q;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+                : "=r"(both_ok)
+                : "r"((uint32_t)ok), "r"(pair_bar)
+                : "memory");
+            if (!both_ok) {
+                ok = false;
+                break;
+            }
+            bm = fmaxf(bm, s_rowmax[hc ^ 1][r]);
+            // both have read before either writes the next block's value
+            asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
             const float mn = fmaxf(m, bm);
             const float msafe = mn == -INFINITY ? 0.f : mn;   // rows with nothing visible yet
             const float corr = exp2f(m - msafe);
@@ -281,23 +304,23 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             // P row r as two bf16 terms, 128-byte swizzled rows (16-byte piece i at i ^ (r % 8))
             uint8_t *prow = pbase + r * 128;
 #pragma unroll
-            for (int piece = 0; piece < AT_KEYS / 8; ++piece) {
+            for (int pc = 0; pc < HK / 8; ++pc) {
                 uint32_t w0[4], w1[4];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                    const float p0 = exp2f(sv[piece * 8 + 2 * e] - msafe);
-                    const float p1 = exp2f(sv[piece * 8 + 2 * e + 1] - msafe);
+                    const float p0 = exp2f(sv[pc * 8 + 2 * e] - msafe);
+                    const float p1 = exp2f(sv[pc * 8 + 2 * e + 1] - msafe);
                     ps += p0 + p1;
                     const uint16_t a0 = f32_to_bf16(p0), b0 = f32_to_bf16(p1);
                     const uint16_t a1 = f32_to_bf16(p0 - bf16_to_f32(a0)), b1 = f32_to_bf16(p1 - bf16_to_f32(b0));
                     w0[e] = (uint32_t)a0 | ((uint32_t)b0 << 16);
                     w1[e] = (uint32_t)a1 | ((uint32_t)b1 << 16);
                 }
-                const int sp = (piece ^ (r & 7)) * 16;
+                const int sp = ((hc * (HK / 8) + pc) ^ (r & 7)) * 16;
                 *reinterpret_cast<uint4 *>(prow + sp) = make_uint4(w0[0], w0[1], w0[2], w0[3]);
                 *reinterpret_cast<uint4 *>(prow + L::P_BYTES + sp) = make_uint4(w1[0], w1[1], w1[2], w1[3]);
             }
-            l = l * corr + ps;
+            l = l * corr + ps;        // this half's share of the row sum, in the shared scale
             m = mn;
             fence_proxy_async_smem();   // generic-proxy writes of P before the MMA reads them
             tc_fence_before();
@@ -310,11 +333,16 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             corr_prev = corr;
         }
         if (ok && nb > 0) fold(nb - 1, corr_prev);
+        // the row sum: both halves
+        // the row sum of both halves (the last maxima were read before the pair's last barrier)
+        s_rowmax[hc][r] = l;
+        asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
+        l += s_rowmax[hc ^ 1][r];
         if (ok && row_ok && tok < a.T) {
             const float inv = 1.0f / l;
-            const size_t off = (size_t)tok * a.nq * D + (size_t)head * D;
+            const size_t off = (size_t)tok * a.nq * D + (size_t)head * D + hc * HD;
 #pragma unroll
-            for (int c = 0; c < D; c += 8) {
+            for (int c = 0; c < HD; c += 8) {
                 uint32_t w0[4], w1[4], w2[4];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {

@@ -197,6 +197,40 @@ __device__ __forceinline__ float dot8(const uint4 w, const float *h, float a) {
     return a;
 }
 
+// Warp sums of a slot's RPS rows (each lane holds its partial of every row),
+// stored to rb[0, rows): a transposed butterfly.  R = RPS rounded up to a power
+// of two; at each of the first log2(R) levels a lane keeps one half of its rows
+// and trades the other half with its partner, so one shuffle moves one row (R - 1
+// shuffles in all instead of 5 R); plain butterflies finish the sum.  Lane l then
+// holds the row whose index is spelled by lane bits 4, 3, ... (most significant
+// first), and the lanes whose remaining low bits are zero store it.
+template <int RPS>
+__device__ __forceinline__ void warp_rows_store(const float (&acc)[RPS], float *rb, int rows, int lane) {
+    constexpr int R = RPS <= 1 ? 1 : RPS <= 2 ? 2 : RPS <= 4 ? 4 : 8;
+    static_assert(RPS <= 8, "at most 8 rows per slot");
+    float v[R];
+#pragma unroll
+    for (int i = 0; i < R; ++i) v[i] = i < RPS ? acc[i] : 0.f;
+    int row = 0;
+#pragma unroll
+    for (int o = 16, cnt = R; o > 0; o >>= 1) {
+        if (cnt > 1) {
+            const bool up = (lane & o) != 0;
+#pragma unroll
+            for (int t = 0; t < cnt / 2; ++t) {
+                const float send = up ? v[t] : v[t + cnt / 2];
+                const float keep = up ? v[t + cnt / 2] : v[t];
+                v[t] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+            }
+            if (up) row += cnt / 2;
+            cnt >>= 1;
+        } else {
+            v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+        }
+    }
+    if ((lane & (32 / R - 1)) == 0 && row < rows) rb[row] = v[0];
+}
+
 // ------------------------------------------------- 8-bit block rows (decode) --
 // A row of the 8-bit block format in shared memory: K int8 codes (two's
 // complement), then the row's K/32 fp16 block scales.
@@ -1043,16 +1077,7 @@ __device__ bool mc_gemv(MegaRing &R, float *red, int K, int n_units, int rpu, co
         __syncwarp();
         if (lane == 0) mbar_arrive(R.empty0 + 8 * slot);
         ++R.n;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-            for (int r = 0; r < RPS; ++r) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
-        if (lane == 0) {
-            float *rb = red + (size_t)(buf * kGemvWarps + warp) * kRedRows + brow;
-#pragma unroll
-            for (int r = 0; r < RPS; ++r)
-                if (r < rows) rb[r] = acc[r];
-        }
+        warp_rows_store<RPS>(acc, red + (size_t)(buf * kGemvWarps + warp) * kRedRows + brow, rows, lane);
         brow += rows;
         if (s == nst - 1 || brow + RPS > kRedRows) {
             if (consumer_sync_or(!ok)) return false;
@@ -1225,16 +1250,7 @@ __device__ bool mc_gemv_q8(MegaRing &R, float *red, int K, int n_units, int rpu,
         __syncwarp();
         if (lane == 0) mbar_arrive(R.empty0 + 8 * slot);
         ++R.n;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-            for (int r = 0; r < RPS; ++r) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
-        if (lane == 0) {
-            float *rb = red + (size_t)(buf * kGemvWarps + warp) * kRedRows + brow;
-#pragma unroll
-            for (int r = 0; r < RPS; ++r)
-                if (r < rows) rb[r] = acc[r];
-        }
+        warp_rows_store<RPS>(acc, red + (size_t)(buf * kGemvWarps + warp) * kRedRows + brow, rows, lane);
         brow += rows;
         if (s == nst - 1 || brow + RPS > kRedRows) {
             if (consumer_sync_or(!ok)) return false;

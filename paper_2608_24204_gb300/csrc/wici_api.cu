@@ -706,19 +706,9 @@ struct EventHook : LaunchHook {
     }
 };
 
-int wici_profile_decode(wici_ctx *c, int32_t n_steps, const char **names, int32_t *launches, double *total_ms,
-                        int32_t cap, int32_t *n_kinds) {
-    if (!c) return fail(nullptr, WICI_E_ARG, "null context");
-    if (n_steps < 1 || !names || !launches || !total_ms || !n_kinds || cap < 1)
-        return fail(c, WICI_E_ARG, "bad profile arguments");
-    if (int rc = begin_decode(c, n_steps, -1)) return rc;
-    EventHook hook;
-    hook.st = c->stream;
-    for (int i = 0; i < n_steps; ++i) {
-        cudaError_t e = enqueue_decode_step(c->plan, c->bufs, c->stream, false, &hook);
-        if (e != cudaSuccess) return fail(c, WICI_E_CUDA, "profile launch: %s", cudaGetErrorString(e));
-    }
-    int rc = finish_call(c, c->kv_len + n_steps, nullptr);
+// per-kind launches and milliseconds of a finished EventHook into the caller's arrays
+static void report_hook(EventHook &hook, const char **names, int32_t *launches, double *total_ms, int32_t cap,
+                        int32_t *n_kinds) {
     std::vector<double> ms(hook.names.size(), 0.0);
     std::vector<int> cnt(hook.names.size(), 0);
     for (size_t i = 0; i < hook.which.size(); ++i) {
@@ -742,6 +732,49 @@ int wici_profile_decode(wici_ctx *c, int32_t n_steps, const char **names, int32_
         total_ms[i] = ms[i];
     }
     *n_kinds = k;
+}
+
+int wici_profile_decode(wici_ctx *c, int32_t n_steps, const char **names, int32_t *launches, double *total_ms,
+                        int32_t cap, int32_t *n_kinds) {
+    if (!c) return fail(nullptr, WICI_E_ARG, "null context");
+    if (n_steps < 1 || !names || !launches || !total_ms || !n_kinds || cap < 1)
+        return fail(c, WICI_E_ARG, "bad profile arguments");
+    if (int rc = begin_decode(c, n_steps, -1)) return rc;
+    EventHook hook;
+    hook.st = c->stream;
+    for (int i = 0; i < n_steps; ++i) {
+        cudaError_t e = enqueue_decode_step(c->plan, c->bufs, c->stream, false, &hook);
+        if (e != cudaSuccess) return fail(c, WICI_E_CUDA, "profile launch: %s", cudaGetErrorString(e));
+    }
+    int rc = finish_call(c, c->kv_len + n_steps, nullptr);
+    report_hook(hook, names, launches, total_ms, cap, n_kinds);
+    return rc;
+}
+
+int wici_profile_prefill(wici_ctx *c, const int32_t *tokens, int32_t n, const char **names, int32_t *launches,
+                         double *total_ms, int32_t cap, int32_t *n_kinds) {
+    if (!c) return fail(nullptr, WICI_E_ARG, "null context");
+    if (!tokens || n < 1 || !names || !launches || !total_ms || !n_kinds || cap < 1)
+        return fail(c, WICI_E_ARG, "bad profile arguments");
+    if (int rc = check_ready(c)) return rc;
+    const Plan &p = c->plan;
+    if ((int64_t)c->kv_len + n > p.cfg.max_tokens)
+        return fail(c, WICI_E_CAPACITY, "kv_len %d + %d tokens exceeds max_tokens %d", c->kv_len, n,
+                    p.cfg.max_tokens);
+    for (int i = 0; i < n; ++i)
+        if (tokens[i] < 0 || tokens[i] >= p.V) return fail(c, WICI_E_ARG, "token %d out of range", tokens[i]);
+    EventHook hook;
+    hook.st = c->stream;
+    for (int off = 0; off < n; off += p.max_chunk) {
+        const int T = n - off < p.max_chunk ? n - off : p.max_chunk;
+        CUDA_TRY(c, cudaMemcpyAsync(c->bufs.tok, tokens + off, (size_t)T * 4, cudaMemcpyHostToDevice, c->stream));
+        const bool last = off + T == n;
+        CUDA_TRY(c, enqueue_prefill_chunk(p, c->bufs, c->maps, c->stream, c->kv_len + off, T, last ? n : 0, &hook));
+        if (!last) CUDA_TRY(c, cudaStreamSynchronize(c->stream));
+    }
+    int rc = finish_call(c, c->kv_len + n, nullptr);
+    if (rc == WICI_OK) c->prefilled = true;
+    report_hook(hook, names, launches, total_ms, cap, n_kinds);
     return rc;
 }
 

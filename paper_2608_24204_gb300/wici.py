@@ -25,7 +25,7 @@ EXPORTS = ("wici_get_sizes", "wici_create", "wici_load_weights", "wici_load_weig
            "wici_decode", "wici_reset", "wici_set_page_table", "wici_kv_len", "wici_last_error",
            "wici_profile_decode", "wici_check_bounded_wait", "wici_destroy", "wici_lm_head_argmax_noalloc",
            "wici_conv_workspace_bytes", "wici_conv_forward", "wici_conv_backward_data", "wici_conv_backward_filter",
-           "wici_conv_status")
+           "wici_conv_status", "wici_profile_prefill")
 
 
 class wici_config(ctypes.Structure):
@@ -81,6 +81,8 @@ def lib():
         L.wici_last_error.restype = ctypes.c_char_p
         L.wici_profile_decode.argtypes = [vp, i32, P(ctypes.c_char_p), P(i32), P(ctypes.c_double), i32, P(i32)]
         L.wici_check_bounded_wait.argtypes = [vp, i64]
+        L.wici_profile_prefill.argtypes = [vp, P(i32), i32, P(ctypes.c_char_p), P(i32), P(ctypes.c_double), i32,
+                                           P(i32)]
         L.wici_destroy.argtypes = [vp]
         L.wici_destroy.restype = None
         L.wici_lm_head_argmax_noalloc.argtypes = [vp, vp, vp, vp, i32, i32, ctypes.c_float, vp, vp]
@@ -95,7 +97,7 @@ def lib():
                      "wici_decode", "wici_reset", "wici_set_page_table", "wici_profile_decode",
                      "wici_check_bounded_wait", "wici_lm_head_argmax_noalloc", "wici_conv_workspace_bytes",
                      "wici_conv_forward", "wici_conv_backward_data", "wici_conv_backward_filter",
-                     "wici_conv_status"):
+                     "wici_conv_status", "wici_profile_prefill"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -211,6 +213,16 @@ def wici_profile_decode(ctx, n_steps: int, cap: int = 16) -> dict:
     ms = (ctypes.c_double * cap)()
     n = ctypes.c_int32()
     _check(lib().wici_profile_decode(ctx, n_steps, names, launches, ms, cap, ctypes.byref(n)), ctx)
+    return {names[i].decode(): (int(launches[i]), float(ms[i])) for i in range(n.value)}
+
+
+def wici_profile_prefill(ctx, tokens: np.ndarray, cap: int = 16) -> dict:
+    tok = np.ascontiguousarray(tokens, np.int32)
+    names = (ctypes.c_char_p * cap)()
+    launches = (ctypes.c_int32 * cap)()
+    ms = (ctypes.c_double * cap)()
+    n = ctypes.c_int32()
+    _check(lib().wici_profile_prefill(ctx, _i32p(tok), len(tok), names, launches, ms, cap, ctypes.byref(n)), ctx)
     return {names[i].decode(): (int(launches[i]), float(ms[i])) for i in range(n.value)}
 
 

@@ -26,7 +26,7 @@ def declared_entry_points():
 
 def test_library_exports_every_declared_entry_point():
     names = declared_entry_points()
-    assert len(names) == 20
+    assert len(names) == 21
     L = wici.lib()
     for n in names:
         assert hasattr(L, n), n
