@@ -50,12 +50,12 @@ constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;                      // 16 KB
 constexpr uint32_t TC_TMEM_COLS = 512;                                  // two accumulator buffers
 constexpr size_t TC_SMEM_BUDGET = 216 * 1024;                           // ring bytes
 
-// geometry of a 128 x BN output tile
-template <int BN>
+// geometry of a 128 x BN output tile whose stages hold AT activation terms
+template <int BN, int AT = kTerms>
 struct TcTile {
     static_assert(BN % 64 == 0 && BN <= 256, "BN: a multiple of 64 up to 256");
     static constexpr uint32_t B_BYTES = BN * TC_BK * 2;
-    static constexpr uint32_t STAGE_BYTES = kTerms * TC_A_BYTES + B_BYTES;
+    static constexpr uint32_t STAGE_BYTES = AT * TC_A_BYTES + B_BYTES;
     static constexpr int STAGES = (int)(TC_SMEM_BUDGET / STAGE_BYTES);
     static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024;
     static constexpr int EPI_COLS = BN / 2;                               // columns per epilogue warp
@@ -136,10 +136,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                    const __grid_constant__ CUtensorMap map_w1, const __grid_constant__ CUtensorMap map_w2, int T,
                    int N, int K, int *err, const Epi epi) {
     static_assert(WT == 1 || WT == kTerms, "one exact bf16 weight term, or three");
-    // activation terms multiplied against a bf16 weight: the epilogue type states it
-    constexpr int AT = Epi::kATerms;
+    constexpr int AT = Epi::kATerms;   // activation terms multiplied (and loaded)
     static_assert(AT >= 1 && AT <= kTerms, "activation terms");
-    using G = TcTile<BN>;
+    using G = TcTile<BN, AT>;
     constexpr int S = G::STAGES;
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full_bar[S], empty_bar[S], acc_full[2], acc_free[2];
@@ -197,7 +196,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     tma_load_2d(st, &map_a0, kb * TC_BK, m0, fb);
                     if (na > 1) tma_load_2d(st + TC_A_BYTES, &map_a1, kb * TC_BK, m0, fb);
                     if (na > 2) tma_load_2d(st + 2 * TC_A_BYTES, &map_a2, kb * TC_BK, m0, fb);
-                    tma_load_2d(st + kTerms * TC_A_BYTES, j == 0 ? &map_w : j == 1 ? &map_w1 : &map_w2, kb * TC_BK, n0,
+                    tma_load_2d(st + AT * TC_A_BYTES, j == 0 ? &map_w : j == 1 ? &map_w1 : &map_w2, kb * TC_BK, n0,
                                 fb);
                     s_issued = it + 1;
                 }
@@ -225,7 +224,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         const int nt = WT == 1 ? AT : AT - kk / nk;   // activation terms meeting this weight term
                         const uint32_t st = base + (uint32_t)s * G::STAGE_BYTES;
                         // descriptors of k-step 0; each k-step of 16 elements is 32 bytes further
-                        const uint64_t bd0 = tc_desc_sw128(st + kTerms * TC_A_BYTES);
+                        const uint64_t bd0 = tc_desc_sw128(st + AT * TC_A_BYTES);
                         const uint64_t ad0 = tc_desc_sw128(st);
 #pragma unroll
                         for (int k = 0; k < TC_BK / 16; ++k)

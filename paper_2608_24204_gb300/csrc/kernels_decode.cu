@@ -235,10 +235,11 @@ __device__ __forceinline__ void warp_rows_store(const float (&acc)[RPS], float *
 // A row of the 8-bit block format in shared memory: K int8 codes (two's
 // complement), then the row's K/32 fp16 block scales.
 //
-// The input vector of a phase is put once into 24-bit fixed point,
-// X[c] = rint(h[c] * 2^E) with |X| < 2^23 (E from the vector's largest
-// magnitude, one rounding of at most 2^-24 of it), and X is cut into three
-// byte digits X = 65536 X2 + 256 X1 + X0 (X2 signed, X1 and X0 unsigned).  The
+// The input vector of a phase is put once into fixed point, X[c] = rint(h[c] *
+// 2^E) with |X| < 2^23 (three byte digits) or 2^15 (two), E from the vector's
+// largest magnitude (one rounding of at most 2^-24, or 2^-16, of it), and X is
+// cut into byte digits, e.g. X = 65536 X2 + 256 X1 + X0 (X2 signed, the others
+// unsigned).  The
 // integer dot products of 16 codes with each digit (dp4a, exact in int32) make
 // the chunk's exact sum q . X, which one fp32 rounding carries into the row's
 // fp32 accumulator with the block scale; 2^-E is applied once per row.  That is
@@ -1104,10 +1105,12 @@ __device__ bool mc_gemv(MegaRing &R, float *red, int K, int n_units, int rpu, co
 // One GEMV phase over a matrix in the 8-bit block format (rows of
 // q8_row_bytes(K) bytes), same role as mc_gemv.  Thread t owns the 16-element
 // chunks c = t + 256 j of the input, as byte digits of its fixed-point form.
-template <class QS, class Epi>
+// ND: byte digits of the fixed-point input (3: 24 bits; 2: 16 bits)
+template <class QS, int ND, class Epi>
 __device__ bool mc_gemv_q8(MegaRing &R, float *red, int K, int n_units, int rpu, const float *in,
                            const uint16_t *gain, const uint16_t *embed, float *x_out, float eps, int *ctrl, Epi &epi,
                            float *s_part) {
+    static_assert(ND == 2 || ND == 3, "two or three input digits");
     constexpr int NCH = QS::NCH, RPS = QS::RPS;
     constexpr bool FULL = QS::FULL;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -1152,14 +1155,10 @@ __device__ bool mc_gemv_q8(MegaRing &R, float *red, int K, int n_units, int rpu,
             for (int e = 0; e < 16; ++e) h[j][e] = 0.f;
         }
     }
+    // with the RMSNorm gain applied (before the common factor 1/rms), and the
+    // largest magnitude for the fixed point: one reduction of (sum of squares, max)
+    float mx = 0.f;
     if (gain) {
-        ss = warp_sum(ss);
-        if (lane == 0) s_part[warp] = ss;
-        consumer_sync();
-        float tot = 0.f;
-#pragma unroll
-        for (int w = 0; w < kGemvWarps; ++w) tot += s_part[w];
-        const float rinv = 1.0f / sqrtf(tot / (float)K + eps);
 #pragma unroll
         for (int j = 0; j < NCH; ++j) {
             const int c = tid + kGemvConsumers * j;
@@ -1170,42 +1169,58 @@ __device__ bool mc_gemv_q8(MegaRing &R, float *red, int K, int n_units, int rpu,
                     const float gg[8] = {bf16lo(gw.x), bf16hi(gw.x), bf16lo(gw.y), bf16hi(gw.y),
                                          bf16lo(gw.z), bf16hi(gw.z), bf16lo(gw.w), bf16hi(gw.w)};
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) h[j][hv * 8 + e] = h[j][hv * 8 + e] * rinv * gg[e];
+                    for (int e = 0; e < 8; ++e) h[j][hv * 8 + e] *= gg[e];
                 }
             }
         }
     }
-    // fixed point: M * 2^E in [2^22, 2^23) for the largest magnitude M
-    float mx = 0.f;
 #pragma unroll
     for (int j = 0; j < NCH; ++j)
 #pragma unroll
         for (int e = 0; e < 16; ++e) mx = fmaxf(mx, fabsf(h[j][e]));
+    ss = warp_sum(ss);
     mx = warp_max(mx);
-    consumer_sync();   // the RMSNorm reads of s_part are done
-    if (lane == 0) s_part[warp] = mx;
+    if (lane == 0) {
+        s_part[warp] = ss;
+        s_part[kGemvWarps + warp] = mx;
+    }
     consumer_sync();
-    float M = 0.f;
+    float tot = 0.f, M = 0.f;
 #pragma unroll
-    for (int w = 0; w < kGemvWarps; ++w) M = fmaxf(M, s_part[w]);
-    const int E = M > 0.f ? min(22 - ilogbf(M), 120) : 0;
+    for (int w = 0; w < kGemvWarps; ++w) {
+        tot += s_part[w];
+        M = fmaxf(M, s_part[kGemvWarps + w]);
+    }
+    if (gain) {
+        const float rinv = 1.0f / sqrtf(tot / (float)K + eps);
+        M *= rinv;
+#pragma unroll
+        for (int j = 0; j < NCH; ++j)
+#pragma unroll
+            for (int e = 0; e < 16; ++e) h[j][e] *= rinv;
+    }
+    // fixed point: M * 2^E just below 2^(8 ND - 1) for the largest magnitude M
+    // (values that round past the limit are clamped to it)
+    constexpr int XBITS = 8 * ND - 1;
+    const int E = M > 0.f ? min(XBITS - 1 - ilogbf(M), 120) : 0;
     const float to_fixed = ldexpf(1.0f, E), from_fixed = ldexpf(1.0f, -E);
-    uint32_t dg[NCH][3][4];   // [chunk][digit X2, X1, X0][4 words of 4 byte digits]
+    // byte digits, most significant (signed) first: X = sum_i X_i 256^(ND-1-i)
+    uint32_t dg[NCH][ND][4];   // [chunk][digit][4 words of 4 byte digits]
 #pragma unroll
     for (int j = 0; j < NCH; ++j)
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            uint32_t w2 = 0, w1 = 0, w0 = 0;
+            uint32_t w[ND];
+#pragma unroll
+            for (int i = 0; i < ND; ++i) w[i] = 0;
 #pragma unroll
             for (int b = 0; b < 4; ++b) {
-                const int X = max(min(__float2int_rn(h[j][4 * k + b] * to_fixed), (1 << 23) - 1), -(1 << 23) + 1);
-                w2 |= ((uint32_t)(X >> 16) & 0xFFu) << (8 * b);
-                w1 |= ((uint32_t)(X >> 8) & 0xFFu) << (8 * b);
-                w0 |= ((uint32_t)X & 0xFFu) << (8 * b);
+                const int X = max(min(__float2int_rn(h[j][4 * k + b] * to_fixed), (1 << XBITS) - 1), -(1 << XBITS) + 1);
+#pragma unroll
+                for (int i = 0; i < ND; ++i) w[i] |= ((uint32_t)(X >> (8 * (ND - 1 - i))) & 0xFFu) << (8 * b);
             }
-            dg[j][0][k] = w2;
-            dg[j][1][k] = w1;
-            dg[j][2][k] = w0;
+#pragma unroll
+            for (int i = 0; i < ND; ++i) dg[j][i][k] = w[i];
         }
 
     const uint32_t row_bytes = (uint32_t)q8_row_bytes((size_t)K);
@@ -1234,16 +1249,18 @@ __device__ bool mc_gemv_q8(MegaRing &R, float *red, int K, int n_units, int rpu,
                         if (j < NCH - 1 || tail_ok) {
                             const uint4 w = lds128(sb + r * row_bytes + j * kGemvConsumers * 16);
                             const float d = lds_f16(sc + r * row_bytes + j * (kGemvConsumers / 2) * 2);
-                            int a2 = dp4a_ss(w.x, dg[j][0][0], 0), a1 = dp4a_su(w.x, dg[j][1][0], 0),
-                                a0 = dp4a_su(w.x, dg[j][2][0], 0);
-                            a2 = dp4a_ss(w.y, dg[j][0][1], a2); a1 = dp4a_su(w.y, dg[j][1][1], a1);
-                            a0 = dp4a_su(w.y, dg[j][2][1], a0);
-                            a2 = dp4a_ss(w.z, dg[j][0][2], a2); a1 = dp4a_su(w.z, dg[j][1][2], a1);
-                            a0 = dp4a_su(w.z, dg[j][2][2], a0);
-                            a2 = dp4a_ss(w.w, dg[j][0][3], a2); a1 = dp4a_su(w.w, dg[j][1][3], a1);
-                            a0 = dp4a_su(w.w, dg[j][2][3], a0);
-                            const float cv = fmaf(small_int_to_f32(a2), 65536.0f,
-                                                  fmaf(small_int_to_f32(a1), 256.0f, small_int_to_f32(a0)));
+                            const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+                            int a[ND];
+#pragma unroll
+                            for (int i = 0; i < ND; ++i) a[i] = 0;
+#pragma unroll
+                            for (int k = 0; k < 4; ++k)
+#pragma unroll
+                                for (int i = 0; i < ND; ++i)
+                                    a[i] = i == 0 ? dp4a_ss(ws[k], dg[j][i][k], a[i]) : dp4a_su(ws[k], dg[j][i][k], a[i]);
+                            float cv = small_int_to_f32(a[0]);
+#pragma unroll
+                            for (int i = 1; i < ND; ++i) cv = fmaf(cv, 256.0f, small_int_to_f32(a[i]));
                             acc[r] = fmaf(d, cv, acc[r]);
                         }
         }
@@ -1274,13 +1291,20 @@ __device__ bool mc_gemv_q8(MegaRing &R, float *red, int K, int n_units, int rpu,
     return true;
 }
 
+// Input digits of the 8-bit GEMV phases: three (24 bits) for QKV, whose outputs
+// become the bf16 K/V and the queries, and kQ8RestDigits for O, gate/up, down.
+#ifndef WICI_Q8_REST_DIGITS
+#define WICI_Q8_REST_DIGITS 3
+#endif
+constexpr int kQ8QkvDigits = 3, kQ8RestDigits = WICI_Q8_REST_DIGITS;
+
 // a per-layer GEMV phase in the layer matrices' format
-template <bool Q8, class S, class Epi>
+template <bool Q8, class S, int ND = kQ8RestDigits, class Epi>
 __device__ __forceinline__ bool mc_layer_gemv(MegaRing &R, float *red, int K, int n_units, int rpu, const float *in,
                                               const uint16_t *gain, const uint16_t *embed, float *x_out, float eps,
                                               int *ctrl, Epi &epi, float *s_part) {
     if constexpr (Q8)
-        return mc_gemv_q8<S>(R, red, K, n_units, rpu, in, gain, embed, x_out, eps, ctrl, epi, s_part);
+        return mc_gemv_q8<S, ND>(R, red, K, n_units, rpu, in, gain, embed, x_out, eps, ctrl, epi, s_part);
     else
         return mc_gemv<S>(R, red, K, n_units, rpu, in, gain, embed, x_out, eps, ctrl, epi, s_part);
 }
@@ -1589,7 +1613,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
     float *red = reinterpret_cast<float *>(smem);
     __shared__ __align__(8) uint64_t bars[2 * kMegaSlots];
     __shared__ __align__(16) float s_state[kFdMaxQueryWarps][D + 4];
-    __shared__ float s_part[kGemvWarps];
+    __shared__ float s_part[2 * kGemvWarps];  // per-warp partials: sums, then maxima (8-bit phases)
     __shared__ float s_bv[kGemvWarps];
     __shared__ int s_bi[kGemvWarps];
     __shared__ int s_flag, s_last, s_abort;
@@ -1655,7 +1679,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) decode_step_kernel(const Mega
         eq.bias = a.bias ? a.W + a.l0.bqkv + lo : nullptr;
         eq.kraw = a.kraw;
         eq.qdim = a.qdim; eq.kvdim = a.kvdim; eq.d = a.d; eq.nkv = a.nkv; eq.page_elems = a.page_elems;
-        ok = mc_layer_gemv<Q8, LH>(R, red, a.H, a.nqkv / 2, 2, a.x, a.W + a.l0.attn_norm + lo,
+        ok = mc_layer_gemv<Q8, LH, kQ8QkvDigits>(R, red, a.H, a.nqkv / 2, 2, a.x, a.W + a.l0.attn_norm + lo,
                                    l == 0 ? a.W + a.w_embed : nullptr, a.x, a.eps, a.ctrl, eq, s_part) &&
              mega_grid_sync(a.ctrl, ++k, &s_flag);
         if (!ok) break;

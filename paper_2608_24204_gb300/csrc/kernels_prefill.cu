@@ -490,27 +490,22 @@ const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
     }
     static bool attrs = false;
     if (!attrs) {
-        constexpr int s192 = (int)TcTile<192>::SMEM, s128 = (int)TcTile<128>::SMEM;
         const auto attr = [](const void *f, int bytes) {
             return cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) == cudaSuccess;
         };
-        if (!attr((const void *)gemm_tc_kernel<192, 1, PEpiQKV>, s192) ||
-            !attr((const void *)gemm_tc_kernel<192, 1, PEpiResidual>, s192) ||
-            !attr((const void *)gemm_tc_kernel<192, 1, PEpiSwiGLU>, s192) ||
-            !attr((const void *)gemm_tc_kernel<128, 1, PEpiQKV>, s128) ||
-            !attr((const void *)gemm_tc_kernel<128, 1, PEpiResidual>, s128) ||
-            !attr((const void *)gemm_tc_kernel<128, 1, PEpiSwiGLU>, s128) ||
-            !attr((const void *)gemm_tc_kernel<192, kTerms, PEpiQKV>, s192) ||
-            !attr((const void *)gemm_tc_kernel<192, kTerms, PEpiResidual>, s192) ||
-            !attr((const void *)gemm_tc_kernel<192, kTerms, PEpiSwiGLU>, s192) ||
-            !attr((const void *)gemm_tc_kernel<128, kTerms, PEpiQKV>, s128) ||
-            !attr((const void *)gemm_tc_kernel<128, kTerms, PEpiResidual>, s128) ||
-            !attr((const void *)gemm_tc_kernel<128, kTerms, PEpiSwiGLU>, s128) ||
+#define WICI_GEMM_ATTR(BN, WT, E) attr((const void *)gemm_tc_kernel<BN, WT, E>, (int)TcTile<BN, E::kATerms>::SMEM)
+        if (!WICI_GEMM_ATTR(192, 1, PEpiQKV) || !WICI_GEMM_ATTR(192, 1, PEpiResidual) ||
+            !WICI_GEMM_ATTR(192, 1, PEpiSwiGLU) || !WICI_GEMM_ATTR(128, 1, PEpiQKV) ||
+            !WICI_GEMM_ATTR(128, 1, PEpiResidual) || !WICI_GEMM_ATTR(128, 1, PEpiSwiGLU) ||
+            !WICI_GEMM_ATTR(192, kTerms, PEpiQKV) || !WICI_GEMM_ATTR(192, kTerms, PEpiResidual) ||
+            !WICI_GEMM_ATTR(192, kTerms, PEpiSwiGLU) || !WICI_GEMM_ATTR(128, kTerms, PEpiQKV) ||
+            !WICI_GEMM_ATTR(128, kTerms, PEpiResidual) || !WICI_GEMM_ATTR(128, kTerms, PEpiSwiGLU) ||
             cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)(AttnSmem<128>::TOTAL + 1024)) != cudaSuccess ||
             cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)(AttnSmem<64>::TOTAL + 1024)) != cudaSuccess)
             return "cannot raise the shared-memory limit of the tensor-core GEMM";
+#undef WICI_GEMM_ATTR
         attrs = true;
     }
     return nullptr;
@@ -553,10 +548,10 @@ static void launch_gemm(const Plan &p, const CUtensorMap *a, const WOperand &w, 
     const int tiles = ((T + TC_BM - 1) / TC_BM) * ((N + BN - 1) / BN);
     const int grid = tiles < p.num_sms ? tiles : p.num_sms;   // persistent: at most one CTA per SM
     if (w.terms == 1)
-        gemm_tc_kernel<BN, 1, Epi><<<grid, TC_THREADS, TcTile<BN>::SMEM, st>>>(a[0], a[1], a[2], *w.w[0], *w.w[1],
+        gemm_tc_kernel<BN, 1, Epi><<<grid, TC_THREADS, TcTile<BN, Epi::kATerms>::SMEM, st>>>(a[0], a[1], a[2], *w.w[0], *w.w[1],
                                                                               *w.w[2], T, N, K, err, epi);
     else
-        gemm_tc_kernel<BN, kTerms, Epi><<<grid, TC_THREADS, TcTile<BN>::SMEM, st>>>(
+        gemm_tc_kernel<BN, kTerms, Epi><<<grid, TC_THREADS, TcTile<BN, Epi::kATerms>::SMEM, st>>>(
             a[0], a[1], a[2], *w.w[0], *w.w[1], *w.w[2], T, N, K, err, epi);
 }
 
