@@ -6,14 +6,18 @@
 // from the paged cache in blocks of 64 (four 16-key pages, fetched by 5-D TMA
 // through the page table).  Per block j:
 //   S_j  = (Q_0 + Q_1) K_j^T      tcgen05.mma, M=128 rows, N=64 keys, fp32 in TMEM
-//   softmax (one row per thread, read from TMEM): online max/sum, P_j = exp2(s - m_j)
-//   O_j  = (P_0 + P_1) V_j        tcgen05.mma, N=d, V read as an MN-major operand
-//   O = O * exp2(m_{j-1} - m_j) + O_j   in registers
-// S, P and O_j are double-buffered (two TMEM accumulators each for S and O_j, two
-// P tiles in shared memory), so the tensor cores work ahead of the softmax: the
-// MMA warp issues S_{j+2} as soon as the softmax has consumed S_j, and P_j V_j
-// runs while the softmax computes P_{j+1}; the softmax folds O_j into its
-// registers one block late.
+//   softmax (one row per thread pair, read from TMEM): P_j = exp2(s - m), with m
+//          the row's reference maximum
+//   O   += (P_0 + P_1) V_j        tcgen05.mma, N=d, V read as an MN-major operand,
+//          accumulated in TMEM over all blocks
+// The reference maximum only moves when a block's maximum exceeds it by more
+// than 2^8 (so P <= 256): then the softmax rescales its rows of the TMEM
+// accumulator and its row sums by exp2(m_old - m_new), between P_{j-1} V_{j-1}
+// and P_j V_j; the result O / l is the same softmax in exact arithmetic.
+// S and P are double-buffered (two TMEM accumulators for S, two P tiles in
+// shared memory), so the tensor cores work ahead of the softmax: the MMA warp
+// issues S_{j+2} as soon as the softmax has consumed S_j, and P_j V_j runs while
+// the softmax computes P_{j+1}.
 // Q and P are carried as two bf16 terms (hi + lo: 16 significant bits), K and V
 // are exact bf16: the products only meet bf16 K and V, whose own rounding is 2^-9,
 // and the two-term tiles leave room for a three-stage K/V ring.  Warp roles:
@@ -37,7 +41,8 @@ constexpr int AT_KEYS = 64;            // keys per block
 constexpr int AT_STAGES = 3;           // K/V ring depth
 constexpr int AT_TERMS = 2;            // bf16 terms of the Q and P operands
 constexpr int AT_THREADS = 320;     // producer, MMA, 8 softmax warps (two per TMEM lane quadrant)
-constexpr uint32_t AT_TMEM_COLS = 512; // S: [0, 64) and [64, 128); O blocks: [128, 128 + d) and [256, 256 + d)
+constexpr uint32_t AT_TMEM_COLS = 256; // S: [0, 64) and [64, 128); O: [128, 128 + d)
+constexpr float AT_RESCALE_LOG2 = 8.f; // the reference maximum trails the row maximum by at most this
 
 enum : int { SITE_AT_Q = 41, SITE_AT_KVE = 42, SITE_AT_KVF = 43, SITE_AT_S = 44, SITE_AT_P = 45, SITE_AT_O = 46,
              SITE_AT_DRAIN = 47 };
@@ -95,6 +100,37 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// 32 lanes x 32 columns of fp32 into TMEM (this warp's lane quadrant); completes at tc_wait_st
+__device__ __forceinline__ void tc_st32(uint32_t taddr, const float *v) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+        "f"(v[0]), "f"(v[1]), "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7]), "f"(v[8]), "f"(v[9]),
+        "f"(v[10]), "f"(v[11]), "f"(v[12]), "f"(v[13]), "f"(v[14]), "f"(v[15]), "f"(v[16]), "f"(v[17]), "f"(v[18]),
+        "f"(v[19]), "f"(v[20]), "f"(v[21]), "f"(v[22]), "f"(v[23]), "f"(v[24]), "f"(v[25]), "f"(v[26]), "f"(v[27]),
+        "f"(v[28]), "f"(v[29]), "f"(v[30]), "f"(v[31])
+        : "memory");
+}
+__device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+// 2^x (PTX ex2.approx, flush-to-zero): 2^-inf = 0
+__device__ __forceinline__ float fast_exp2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+// two floats -> two bf16 (round to nearest even) in one word, lo in bits 0..15
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    uint32_t w;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(w) : "f"(hi), "f"(lo));
+    return w;
+}
+
 // tokens per 128-row tile: the group's query heads of each token share a tile
 __host__ __device__ constexpr int attn_tokens_per_tile(int group) { return AT_ROWS / group; }
 
@@ -115,7 +151,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                    const AttnArgs a) {
     using L = AttnSmem<D>;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t q_full, kv_full[AT_STAGES], kv_empty[AT_STAGES], s_full[2], p_full[2], o_full[2];
+    __shared__ __align__(8) uint64_t q_full, kv_full[AT_STAGES], kv_empty[AT_STAGES], s_full[2], p_full[2], o_full;
     __shared__ uint32_t s_tmem;
     __shared__ int s_issued;
     __shared__ float s_rowmax[2][AT_ROWS];      // [key half][row]: each block's row maxima, the row sums at the end
@@ -139,8 +175,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&s_full[b]), 1);
             mbar_init(smem_u32(&p_full[b]), 8);
-            mbar_init(smem_u32(&o_full[b]), 1);
         }
+        mbar_init(smem_u32(&o_full), 1);
         fence_barrier_init();
         s_issued = 0;
     }
@@ -154,7 +190,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = s_tmem;
-    // buffer b of S at tmem + 64 b, of the O block at tmem + 128 + 128 b
+    // buffer b of S at tmem + 64 b, the O accumulator at tmem + 128
     const uint32_t tm_s = tmem, tm_o = tmem + 128;
 
     if (warp == 0) {
@@ -216,7 +252,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             if (nb > 1) issue_s(1);
             for (int j = 0; j < nb && ok; ++j) {
                 const int s = j % AT_STAGES, b = j & 1;
-                // P_j written (and S_j read, and O_{j-2} folded) by the softmax
+                // P_j written (and S_j read, and O rescaled if its reference maximum moved) by the softmax
                 ok = mbar_wait(smem_u32(&p_full[b]), (j >> 1) & 1, a.err, SITE_AT_P);
                 if (!ok) break;
                 tc_fence_after();
@@ -228,10 +264,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                     const uint64_t vd = at_desc_mn(vb + 2048u * k, AT_KEYS * 128);
 #pragma unroll
                     for (int t = 0; t < AT_TERMS; ++t)
-                        tc_mma(tm_o + 128u * (uint32_t)b, at_desc_k(pb + t * L::P_BYTES + 32u * k), vd, idesc_o,
-                               (k | t) != 0);
+                        tc_mma(tm_o, at_desc_k(pb + t * L::P_BYTES + 32u * k), vd, idesc_o, (j | k | t) != 0);
                 }
-                tc_commit(smem_u32(&o_full[b]));
+                tc_commit(smem_u32(&o_full));
                 tc_commit(smem_u32(&kv_empty[s]));
                 if (j + 2 < nb) issue_s(j + 2);   // S buffer b was read before P_j was posted
             }
@@ -247,39 +282,30 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         const int head = g * a.group + r % a.group;
         const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
         const uint32_t pair_bar = 1 + qd;          // named barrier of the two warps of this quadrant
-        float o[HD];
-#pragma unroll
-        for (int i = 0; i < HD; ++i) o[i] = 0.f;
-        float m = -INFINITY, l = 0.f, corr_prev = 1.f;
+        // blocks before this one are visible to every row of the tile: no causal mask
+        const int first_masked = a.tpt * a.group == AT_ROWS ? (a.P + t0 + 1) / AT_KEYS : 0;
+        float m = -INFINITY, l = 0.f;   // reference maximum (log2 units) and row sum in its scale
         bool ok = true;
         uint8_t *pbase0 = smem_raw + (base - smem_u32(smem_raw)) + L::OFF_P;
-        // O += the P.V block b of the previous iteration, in the new max's scale
-        auto fold = [&](int jb, float corr) {
-            const int b = jb & 1;
-            ok = ok && mbar_wait(smem_u32(&o_full[b]), (jb >> 1) & 1, a.err, SITE_AT_O);
-            tc_fence_after();
-#pragma unroll
-            for (int c0 = 0; c0 < HD; c0 += 32) {
-                float ov[32];
-                tc_ld32(tm_o + 128u * (uint32_t)b + lane_base + hc * HD + c0, ov);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) o[c0 + i] = fmaf(o[c0 + i], corr, ov[i]);
-            }
-        };
+        const uint32_t tm_orow = tm_o + lane_base + hc * HD;
         for (int j = 0; j < nb; ++j) {
             ok = ok && mbar_wait(smem_u32(&s_full[j & 1]), (j >> 1) & 1, a.err, SITE_AT_S);
             tc_fence_after();
             float sv[HK];
             tc_ld32(tm_s + 64u * (uint32_t)(j & 1) + lane_base + hc * HK, sv);
             uint8_t *pbase = pbase0 + (size_t)(j & 1) * AT_TERMS * L::P_BYTES;
-            float bm = -INFINITY;
+            if (j >= first_masked) {
 #pragma unroll
-            for (int c = 0; c < HK; ++c) {
-                const int key = j * AT_KEYS + hc * HK + c;
-                sv[c] = (row_ok && key <= qpos) ? sv[c] * a.scale_log2 : -INFINITY;
-                bm = fmaxf(bm, sv[c]);
+                for (int c = 0; c < HK; ++c) {
+                    const int key = j * AT_KEYS + hc * HK + c;
+                    if (!(row_ok && key <= qpos)) sv[c] = -INFINITY;
+                }
             }
-            // the row's block maximum over both halves
+            float bm = sv[0];
+#pragma unroll
+            for (int c = 1; c + 1 < HK; c += 2) bm = fmax3(bm, sv[c], sv[c + 1]);
+            if ((HK & 1) == 0) bm = fmaxf(bm, sv[HK - 1]);
+            // the row's block maximum over both halves (raw scores: the scale is positive)
             s_rowmax[hc][r] = bm;
             // the pair leaves the loop together: the barrier also ANDs the two warps'
             // wait results, so a wait that gave up in one warp never strands the other
@@ -294,46 +320,73 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                 ok = false;
                 break;
             }
-            bm = fmaxf(bm, s_rowmax[hc ^ 1][r]);
+            bm = fmaxf(bm, s_rowmax[hc ^ 1][r]) * a.scale_log2;
             // both have read before either writes the next block's value
             asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
-            const float mn = fmaxf(m, bm);
-            const float msafe = mn == -INFINITY ? 0.f : mn;   // rows with nothing visible yet
-            const float corr = exp2f(m - msafe);
+            // a new reference maximum only when this block's exceeds it by more than 2^8
+            const bool grow = bm > m + AT_RESCALE_LOG2;
+            const float mn = grow ? bm : m;
+            const float corr = grow ? fast_exp2(m - mn) : 1.f;
+            const float nms = mn == -INFINITY ? 0.f : -mn;   // rows with nothing visible yet
             float ps = 0.f;
             // P row r as two bf16 terms, 128-byte swizzled rows (16-byte piece i at i ^ (r % 8))
+            uint32_t w0[HK / 2], w1[HK / 2];
+#pragma unroll
+            for (int e = 0; e < HK / 2; ++e) {
+                const float p0 = fast_exp2(fmaf(sv[2 * e], a.scale_log2, nms));
+                const float p1 = fast_exp2(fmaf(sv[2 * e + 1], a.scale_log2, nms));
+                ps += p0 + p1;
+                w0[e] = pack_bf16x2(p0, p1);
+                w1[e] = pack_bf16x2(p0 - bf16lo(w0[e]), p1 - bf16hi(w0[e]));
+            }
+            // buffer j & 1 is free: S_j completing means P_{j-2} V_{j-2} has too
             uint8_t *prow = pbase + r * 128;
 #pragma unroll
             for (int pc = 0; pc < HK / 8; ++pc) {
-                uint32_t w0[4], w1[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float p0 = exp2f(sv[pc * 8 + 2 * e] - msafe);
-                    const float p1 = exp2f(sv[pc * 8 + 2 * e + 1] - msafe);
-                    ps += p0 + p1;
-                    const uint16_t a0 = f32_to_bf16(p0), b0 = f32_to_bf16(p1);
-                    const uint16_t a1 = f32_to_bf16(p0 - bf16_to_f32(a0)), b1 = f32_to_bf16(p1 - bf16_to_f32(b0));
-                    w0[e] = (uint32_t)a0 | ((uint32_t)b0 << 16);
-                    w1[e] = (uint32_t)a1 | ((uint32_t)b1 << 16);
-                }
                 const int sp = ((hc * (HK / 8) + pc) ^ (r & 7)) * 16;
-                *reinterpret_cast<uint4 *>(prow + sp) = make_uint4(w0[0], w0[1], w0[2], w0[3]);
-                *reinterpret_cast<uint4 *>(prow + L::P_BYTES + sp) = make_uint4(w1[0], w1[1], w1[2], w1[3]);
+                *reinterpret_cast<uint4 *>(prow + sp) =
+                    make_uint4(w0[4 * pc], w0[4 * pc + 1], w0[4 * pc + 2], w0[4 * pc + 3]);
+                *reinterpret_cast<uint4 *>(prow + L::P_BYTES + sp) =
+                    make_uint4(w1[4 * pc], w1[4 * pc + 1], w1[4 * pc + 2], w1[4 * pc + 3]);
             }
-            l = l * corr + ps;        // this half's share of the row sum, in the shared scale
+            // O is rescaled once P_{j-1} V_{j-1} has landed and before P_j V_j is issued.
+            // Here o_full has completed j - 1 or j phases (S_j completing implies
+            // P_{j-2} V_{j-2} did; P_j is not posted), so its parity wait is exact even
+            // when earlier iterations skipped it; the last iteration always waits, which
+            // keeps the final wait below exact too.
+            const bool any_grow = __any_sync(0xFFFFFFFFu, grow);
+            if (j > 0 && (any_grow || j == nb - 1)) {
+                ok = ok && mbar_wait(smem_u32(&o_full), (j - 1) & 1, a.err, SITE_AT_O);
+                tc_fence_after();
+                if (any_grow) {
+#pragma unroll
+                    for (int c0 = 0; c0 < HD; c0 += 32) {
+                        float ov[32];
+                        tc_ld32(tm_orow + c0, ov);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) ov[i] *= corr;
+                        tc_st32(tm_orow + c0, ov);
+                    }
+                    tc_wait_st();
+                }
+            }
+            l = l * corr + ps;        // this half's share of the row sum, in the reference scale
             m = mn;
             fence_proxy_async_smem();   // generic-proxy writes of P before the MMA reads them
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&p_full[j & 1]));
-            // fold the previous block, whose P.V ran while this block's P was computed;
-            // this also frees its P tile and O accumulator for block j + 1
-            if (j > 0) fold(j - 1, corr_prev);
-            tc_fence_before();
-            corr_prev = corr;
         }
-        if (ok && nb > 0) fold(nb - 1, corr_prev);
-        // the row sum: both halves
+        // the last P.V: O complete in TMEM
+        float o[HD];
+#pragma unroll
+        for (int i = 0; i < HD; ++i) o[i] = 0.f;
+        if (ok && nb > 0) {
+            ok = mbar_wait(smem_u32(&o_full), (nb - 1) & 1, a.err, SITE_AT_O);
+            tc_fence_after();
+#pragma unroll
+            for (int c0 = 0; c0 < HD; c0 += 32) tc_ld32(tm_orow + c0, o + c0);
+        }
         // the row sum of both halves (the last maxima were read before the pair's last barrier)
         s_rowmax[hc][r] = l;
         asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory");
