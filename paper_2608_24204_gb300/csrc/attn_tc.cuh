@@ -10,22 +10,25 @@
 //          the row's reference maximum
 //   O   += (P_0 + P_1) V_j        tcgen05.mma, N=d, V read as an MN-major operand,
 //          accumulated in TMEM over all blocks
+// Both A operands live in tensor memory: the softmax warps store the tile's Q
+// terms there once, and each block's P terms next to S.  Shared memory then only
+// holds the K/V ring, and the tensor cores read only K and V from it (an N=64
+// MMA that also read its A operand from shared memory would need more than the
+// 128 bytes per clock that shared memory delivers).
 // The reference maximum only moves when a block's maximum exceeds it by more
 // than 2^8 (so P <= 256): then the softmax rescales its rows of the TMEM
 // accumulator and its row sums by exp2(m_old - m_new), between P_{j-1} V_{j-1}
 // and P_j V_j; the result O / l is the same softmax in exact arithmetic.
-// S and P are double-buffered (two TMEM accumulators for S, two P tiles in
-// shared memory), so the tensor cores work ahead of the softmax: the MMA warp
-// issues S_{j+2} as soon as the softmax has consumed S_j, and P_j V_j runs while
-// the softmax computes P_{j+1}.
+// S and P are double-buffered, so the tensor cores work ahead of the softmax:
+// the MMA warp issues S_{j+2} as soon as the softmax has consumed S_j, and
+// P_j V_j runs while the softmax computes P_{j+1}.
 // Q and P are carried as two bf16 terms (hi + lo: 16 significant bits), K and V
-// are exact bf16: the products only meet bf16 K and V, whose own rounding is 2^-9,
-// and the two-term tiles leave room for a three-stage K/V ring.  Warp roles:
-// 0 TMA producer, 1 TMEM owner + MMA issuer, 2..9 softmax / output: two warps
-// per TMEM lane quadrant (warp % 4), one for keys 0..31 and output columns
-// [0, d/2) of its 32 rows, the other for keys 32..63 and columns [d/2, d); the
-// pair exchanges each block's row maxima through shared memory.  Every wait is
-// bounded.
+// are exact bf16: the products only meet bf16 K and V, whose own rounding is 2^-9.
+// Warp roles: 0 TMA producer, 1 TMEM owner + MMA issuer, 2..9 softmax / output:
+// two warps per TMEM lane quadrant (warp % 4), one for keys 0..31, d values
+// [0, d/2) of Q and output columns [0, d/2) of its 32 rows, the other for keys
+// 32..63 and the upper halves; the pair exchanges each block's row maxima
+// through shared memory.  Every wait is bounded.
 #pragma once
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -38,28 +41,33 @@ namespace wici {
 
 constexpr int AT_ROWS = 128;           // query rows per tile (TMEM lanes)
 constexpr int AT_KEYS = 64;            // keys per block
-constexpr int AT_STAGES = 3;           // K/V ring depth
+constexpr int AT_STAGES = 6;           // K/V ring depth
 constexpr int AT_TERMS = 2;            // bf16 terms of the Q and P operands
-constexpr int AT_THREADS = 320;     // producer, MMA, 8 softmax warps (two per TMEM lane quadrant)
-constexpr uint32_t AT_TMEM_COLS = 256; // S: [0, 64) and [64, 128); O: [128, 128 + d)
+constexpr int AT_THREADS = 320;        // producer, MMA, 8 softmax warps (two per TMEM lane quadrant)
+constexpr uint32_t AT_TMEM_COLS = 512;
 constexpr float AT_RESCALE_LOG2 = 8.f; // the reference maximum trails the row maximum by at most this
 
 enum : int { SITE_AT_Q = 41, SITE_AT_KVE = 42, SITE_AT_KVF = 43, SITE_AT_S = 44, SITE_AT_P = 45, SITE_AT_O = 46,
              SITE_AT_DRAIN = 47 };
 
+// TMEM columns (one 32-bit column holds two bf16 of a row): Q terms [0, d),
+// S buffers [d, d + 128), P buffers (two terms of 32 columns each) [d + 128, d + 256),
+// the O accumulator [d + 256, 2d + 256)
+template <int D>
+struct AttnTmem {
+    static constexpr uint32_t Q = 0, S = D, P = D + 128, O = D + 256;
+    static_assert(2 * D + 256 <= (int)AT_TMEM_COLS, "tensor memory");
+};
+
 template <int D>
 struct AttnSmem {
     static constexpr int DCH = D / 64;                                   // 64-element d chunks
-    static constexpr uint32_t Q_BYTES = AT_ROWS * D * 2;                 // one term
     static constexpr uint32_t KV_BYTES = AT_KEYS * D * 2;                // K (or V) of a block
-    static constexpr uint32_t P_BYTES = AT_ROWS * AT_KEYS * 2;           // one term
-    static constexpr uint32_t OFF_Q = 0;                                 // [term]
-    static constexpr uint32_t OFF_KV = AT_TERMS * Q_BYTES;               // [stage][K | V]
-    static constexpr uint32_t OFF_P = OFF_KV + AT_STAGES * 2 * KV_BYTES; // [buffer][term]
-    static constexpr uint32_t TOTAL = OFF_P + 2 * AT_TERMS * P_BYTES;
+    static constexpr uint32_t OFF_KV = 0;                                // [stage][K | V]
+    static constexpr uint32_t TOTAL = AT_STAGES * 2 * KV_BYTES;
 };
 
-// K-major, 128-byte swizzle, 8-row groups 1024 B apart (Q, K and P operands)
+// K-major, 128-byte swizzle, 8-row groups 1024 B apart (the K operand)
 __device__ __forceinline__ uint64_t at_desc_k(uint32_t saddr) { return tc_desc_sw128(saddr); }
 
 // MN-major, 128-byte swizzle (V as the B operand of P.V): rows are keys (the K
@@ -81,13 +89,6 @@ __host__ __device__ constexpr uint32_t at_idesc(int n, bool b_mn) {
            ((uint32_t)(AT_ROWS >> 4) << 24);
 }
 
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, int x, int y, int z, uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-        "l"((uint64_t)map), "r"(x), "r"(y), "r"(z), "r"(bar)
-        : "memory");
-}
-
 __device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap *map, int c0, int c1, int c2, int c3, int c4,
                                             uint32_t bar) {
     asm volatile(
@@ -96,19 +97,41 @@ __device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
-__device__ __forceinline__ void fence_proxy_async_smem() {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
-// 32 lanes x 32 columns of fp32 into TMEM (this warp's lane quadrant); completes at tc_wait_st
-__device__ __forceinline__ void tc_st32(uint32_t taddr, const float *v) {
+// 32 lanes x 32 (16) columns of 32-bit words into TMEM (this warp's lane quadrant); complete at tc_wait_st
+__device__ __forceinline__ void tc_st32(uint32_t taddr, const uint32_t *v) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
         "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
-        "f"(v[0]), "f"(v[1]), "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7]), "f"(v[8]), "f"(v[9]),
-        "f"(v[10]), "f"(v[11]), "f"(v[12]), "f"(v[13]), "f"(v[14]), "f"(v[15]), "f"(v[16]), "f"(v[17]), "f"(v[18]),
-        "f"(v[19]), "f"(v[20]), "f"(v[21]), "f"(v[22]), "f"(v[23]), "f"(v[24]), "f"(v[25]), "f"(v[26]), "f"(v[27]),
-        "f"(v[28]), "f"(v[29]), "f"(v[30]), "f"(v[31])
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+        "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]), "r"(v[17]), "r"(v[18]),
+        "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]),
+        "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+        : "memory");
+}
+__device__ __forceinline__ void tc_st16(uint32_t taddr, const uint32_t *v) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15, %16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+        "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
+}
+template <int N>
+__device__ __forceinline__ void tc_st_cols(uint32_t taddr, const uint32_t *v) {
+    static_assert(N == 16 || N == 32, "16 or 32 columns");
+    if constexpr (N == 32)
+        tc_st32(taddr, v);
+    else
+        tc_st16(taddr, v);
+}
+
+// D (+)= A B with the A operand (M = 128 rows on the TMEM lanes, K-major bf16 pairs) in tensor memory
+__device__ __forceinline__ void tc_mma_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(tmem_d),
+        "r"(tmem_a), "l"(bdesc), "r"(idesc), "r"(accumulate)
         : "memory");
 }
 __device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
@@ -135,6 +158,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 __host__ __device__ constexpr int attn_tokens_per_tile(int group) { return AT_ROWS / group; }
 
 struct AttnArgs {
+    const uint16_t *Q[AT_TERMS];  // [T][nq * d] query terms
     uint16_t *O[kTerms];  // [T][nq * d] output terms
     const int *pages;     // logical -> physical page
     int *err;
@@ -146,12 +170,11 @@ struct AttnArgs {
 
 template <int D>
 __global__ void __launch_bounds__(AT_THREADS, 1)
-    attn_tc_kernel(const __grid_constant__ CUtensorMap map_q0, const __grid_constant__ CUtensorMap map_q1,
-                   const __grid_constant__ CUtensorMap map_kv,
-                   const AttnArgs a) {
+    attn_tc_kernel(const __grid_constant__ CUtensorMap map_kv, const AttnArgs a) {
     using L = AttnSmem<D>;
+    using TM = AttnTmem<D>;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t q_full, kv_full[AT_STAGES], kv_empty[AT_STAGES], s_full[2], p_full[2], o_full;
+    __shared__ __align__(8) uint64_t q_ready, kv_full[AT_STAGES], kv_empty[AT_STAGES], s_full[2], p_full[2], o_full;
     __shared__ uint32_t s_tmem;
     __shared__ int s_issued;
     __shared__ float s_rowmax[2][AT_ROWS];      // [key half][row]: each block's row maxima, the row sums at the end
@@ -164,10 +187,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     const int nkeys = a.P + t_end;                    // keys the tile's last token sees
     const int nb = (nkeys + AT_KEYS - 1) / AT_KEYS;
     const uint32_t base = (smem_u32(smem_raw) + 1023u) & ~1023u;
-    const uint32_t q_bytes_box = 64u * (uint32_t)a.group * (uint32_t)a.tpt * 2u;
 
     if (threadIdx.x == 0) {
-        mbar_init(smem_u32(&q_full), 1);
+        mbar_init(smem_u32(&q_ready), 8);
         for (int s = 0; s < AT_STAGES; ++s) {
             mbar_init(smem_u32(&kv_full[s]), 1);
             mbar_init(smem_u32(&kv_empty[s]), 1);
@@ -190,17 +212,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = s_tmem;
-    // buffer b of S at tmem + 64 b, the O accumulator at tmem + 128
-    const uint32_t tm_s = tmem, tm_o = tmem + 128;
+    const uint32_t tm_q = tmem + TM::Q, tm_s = tmem + TM::S, tm_p = tmem + TM::P, tm_o = tmem + TM::O;
 
     if (warp == 0) {
         if (lane == 0) {  // ----------------------------------------------- TMA producer
-            const uint32_t qb = smem_u32(&q_full);
-            mbar_arrive_expect_tx(qb, (uint32_t)AT_TERMS * L::DCH * q_bytes_box);
-            for (int c = 0; c < L::DCH; ++c) {
-                tma_load_3d(base + L::OFF_Q + c * AT_ROWS * 128, &map_q0, c * 64, g * a.group, t0, qb);
-                tma_load_3d(base + L::OFF_Q + L::Q_BYTES + c * AT_ROWS * 128, &map_q1, c * 64, g * a.group, t0, qb);
-            }
             int issued = 0;
             for (int j = 0; j < nb; ++j) {
                 const int s = j % AT_STAGES;
@@ -229,7 +244,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         if (lane == 0) {  // ----------------------------------------------- MMA issuer
             constexpr uint32_t idesc_s = at_idesc(AT_KEYS, false);
             constexpr uint32_t idesc_o = at_idesc(D, true);
-            bool ok = mbar_wait(smem_u32(&q_full), 0, a.err, SITE_AT_Q);
+            bool ok = mbar_wait(smem_u32(&q_ready), 0, a.err, SITE_AT_Q);
             auto issue_s = [&](int j) {
                 const int s = j % AT_STAGES;
                 ok = ok && mbar_wait(smem_u32(&kv_full[s]), (j / AT_STAGES) & 1, a.err, SITE_AT_KVF);
@@ -239,12 +254,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                 const uint32_t sacc = tm_s + 64u * (uint32_t)(j & 1);
 #pragma unroll
                 for (int k = 0; k < D / 16; ++k) {
-                    const uint32_t off = (uint32_t)(k / 4) * (AT_ROWS * 128) + 32u * (k % 4);
+                    // d values 16k..16k+15: 8 TMEM columns of each Q term, 32 bytes of each K row
                     const uint32_t koff = (uint32_t)(k / 4) * (AT_KEYS * 128) + 32u * (k % 4);
                     const uint64_t bd = at_desc_k(kb + koff);
 #pragma unroll
                     for (int t = 0; t < AT_TERMS; ++t)
-                        tc_mma(sacc, at_desc_k(base + L::OFF_Q + t * L::Q_BYTES + off), bd, idesc_s, (k | t) != 0);
+                        tc_mma_ts(sacc, tm_q + (uint32_t)(t * (D / 2) + 8 * k), bd, idesc_s, (k | t) != 0);
                 }
                 tc_commit(smem_u32(&s_full[j & 1]));
             };
@@ -252,19 +267,18 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             if (nb > 1) issue_s(1);
             for (int j = 0; j < nb && ok; ++j) {
                 const int s = j % AT_STAGES, b = j & 1;
-                // P_j written (and S_j read, and O rescaled if its reference maximum moved) by the softmax
+                // P_j stored (and S_j read, and O rescaled if its reference maximum moved) by the softmax
                 ok = mbar_wait(smem_u32(&p_full[b]), (j >> 1) & 1, a.err, SITE_AT_P);
                 if (!ok) break;
                 tc_fence_after();
                 const uint32_t vb = base + L::OFF_KV + (uint32_t)s * 2 * L::KV_BYTES + L::KV_BYTES;
-                const uint32_t pb = base + L::OFF_P + (uint32_t)b * AT_TERMS * L::P_BYTES;
 #pragma unroll
                 for (int k = 0; k < AT_KEYS / 16; ++k) {
-                    // 16 keys = two 8-key groups of V rows; P columns 16k..16k+15
+                    // 16 keys = two 8-key groups of V rows; P columns 8k..8k+7 of each term
                     const uint64_t vd = at_desc_mn(vb + 2048u * k, AT_KEYS * 128);
 #pragma unroll
                     for (int t = 0; t < AT_TERMS; ++t)
-                        tc_mma(tm_o, at_desc_k(pb + t * L::P_BYTES + 32u * k), vd, idesc_o, (j | k | t) != 0);
+                        tc_mma_ts(tm_o, tm_p + 64u * (uint32_t)b + 32u * t + 8u * k, vd, idesc_o, (j | k | t) != 0);
                 }
                 tc_commit(smem_u32(&o_full));
                 tc_commit(smem_u32(&kv_empty[s]));
@@ -272,9 +286,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             }
         }
     } else {  // ------------------------------------------------------- softmax / output
-        constexpr int HK = AT_KEYS / 2, HD = D / 2;   // keys and output columns per warp of a pair
+        constexpr int HK = AT_KEYS / 2, HD = D / 2;   // keys, d values and output columns per warp of a pair
         const int qd = warp & 3;                   // TMEM lane quadrant
-        const int hc = (warp - 2) >> 2;            // which half of the keys and of the output columns
+        const int hc = (warp - 2) >> 2;            // which half of the keys, of Q and of the output columns
         const int r = qd * 32 + lane;              // tile row
         const bool row_ok = r < a.tpt * a.group;
         const int tok = t0 + r / a.group;          // chunk token of this row
@@ -282,18 +296,38 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         const int head = g * a.group + r % a.group;
         const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
         const uint32_t pair_bar = 1 + qd;          // named barrier of the two warps of this quadrant
+        const size_t row_off = (size_t)tok * a.nq * D + (size_t)head * D + hc * HD;
+        {   // this row's half of the Q terms into TMEM (zeros past the chunk)
+            const bool q_ok = row_ok && tok < a.T;
+#pragma unroll
+            for (int t = 0; t < AT_TERMS; ++t) {
+                uint32_t qw[HD / 2];
+#pragma unroll
+                for (int c = 0; c < HD / 8; ++c) {
+                    const uint4 v = q_ok ? *reinterpret_cast<const uint4 *>(a.Q[t] + row_off + 8 * c)
+                                         : make_uint4(0u, 0u, 0u, 0u);
+                    qw[4 * c] = v.x;
+                    qw[4 * c + 1] = v.y;
+                    qw[4 * c + 2] = v.z;
+                    qw[4 * c + 3] = v.w;
+                }
+                tc_st_cols<HD / 2>(tm_q + lane_base + (uint32_t)(t * (D / 2) + hc * (HD / 2)), qw);
+            }
+            tc_wait_st();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&q_ready));
+        }
         // blocks before this one are visible to every row of the tile: no causal mask
         const int first_masked = a.tpt * a.group == AT_ROWS ? (a.P + t0 + 1) / AT_KEYS : 0;
         float m = -INFINITY, l = 0.f;   // reference maximum (log2 units) and row sum in its scale
         bool ok = true;
-        uint8_t *pbase0 = smem_raw + (base - smem_u32(smem_raw)) + L::OFF_P;
         const uint32_t tm_orow = tm_o + lane_base + hc * HD;
         for (int j = 0; j < nb; ++j) {
             ok = ok && mbar_wait(smem_u32(&s_full[j & 1]), (j >> 1) & 1, a.err, SITE_AT_S);
             tc_fence_after();
             float sv[HK];
             tc_ld32(tm_s + 64u * (uint32_t)(j & 1) + lane_base + hc * HK, sv);
-            uint8_t *pbase = pbase0 + (size_t)(j & 1) * AT_TERMS * L::P_BYTES;
             if (j >= first_masked) {
 #pragma unroll
                 for (int c = 0; c < HK; ++c) {
@@ -329,7 +363,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             const float corr = grow ? fast_exp2(m - mn) : 1.f;
             const float nms = mn == -INFINITY ? 0.f : -mn;   // rows with nothing visible yet
             float ps = 0.f;
-            // P row r as two bf16 terms, 128-byte swizzled rows (16-byte piece i at i ^ (r % 8))
+            // P as two bf16 terms: this half's 32 keys are 16 columns of each term
             uint32_t w0[HK / 2], w1[HK / 2];
 #pragma unroll
             for (int e = 0; e < HK / 2; ++e) {
@@ -339,16 +373,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                 w0[e] = pack_bf16x2(p0, p1);
                 w1[e] = pack_bf16x2(p0 - bf16lo(w0[e]), p1 - bf16hi(w0[e]));
             }
-            // buffer j & 1 is free: S_j completing means P_{j-2} V_{j-2} has too
-            uint8_t *prow = pbase + r * 128;
-#pragma unroll
-            for (int pc = 0; pc < HK / 8; ++pc) {
-                const int sp = ((hc * (HK / 8) + pc) ^ (r & 7)) * 16;
-                *reinterpret_cast<uint4 *>(prow + sp) =
-                    make_uint4(w0[4 * pc], w0[4 * pc + 1], w0[4 * pc + 2], w0[4 * pc + 3]);
-                *reinterpret_cast<uint4 *>(prow + L::P_BYTES + sp) =
-                    make_uint4(w1[4 * pc], w1[4 * pc + 1], w1[4 * pc + 2], w1[4 * pc + 3]);
-            }
+            // P buffer j & 1 is free: S_j completing means P_{j-2} V_{j-2} has too
+            const uint32_t prow = tm_p + 64u * (uint32_t)(j & 1) + lane_base + (uint32_t)hc * (HK / 2);
+            tc_st16(prow, w0);
+            tc_st16(prow + 32, w1);
             // O is rescaled once P_{j-1} V_{j-1} has landed and before P_j V_j is issued.
             // Here o_full has completed j - 1 or j phases (S_j completing implies
             // P_{j-2} V_{j-2} did; P_j is not posted), so its parity wait is exact even
@@ -362,17 +390,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
 #pragma unroll
                     for (int c0 = 0; c0 < HD; c0 += 32) {
                         float ov[32];
+                        uint32_t ow[32];
                         tc_ld32(tm_orow + c0, ov);
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) ov[i] *= corr;
-                        tc_st32(tm_orow + c0, ov);
+                        for (int i = 0; i < 32; ++i) ow[i] = __float_as_uint(ov[i] * corr);
+                        tc_st32(tm_orow + c0, ow);
                     }
-                    tc_wait_st();
                 }
             }
+            tc_wait_st();
             l = l * corr + ps;        // this half's share of the row sum, in the reference scale
             m = mn;
-            fence_proxy_async_smem();   // generic-proxy writes of P before the MMA reads them
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&p_full[j & 1]));
@@ -393,7 +421,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         l += s_rowmax[hc ^ 1][r];
         if (ok && row_ok && tok < a.T) {
             const float inv = 1.0f / l;
-            const size_t off = (size_t)tok * a.nq * D + (size_t)head * D + hc * HD;
 #pragma unroll
             for (int c = 0; c < HD; c += 8) {
                 uint32_t w0[4], w1[4], w2[4];
@@ -406,9 +433,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                     w1[e] = (uint32_t)a1 | ((uint32_t)b1 << 16);
                     w2[e] = (uint32_t)a2 | ((uint32_t)b2 << 16);
                 }
-                *reinterpret_cast<uint4 *>(a.O[0] + off + c) = make_uint4(w0[0], w0[1], w0[2], w0[3]);
-                *reinterpret_cast<uint4 *>(a.O[1] + off + c) = make_uint4(w1[0], w1[1], w1[2], w1[3]);
-                *reinterpret_cast<uint4 *>(a.O[2] + off + c) = make_uint4(w2[0], w2[1], w2[2], w2[3]);
+                *reinterpret_cast<uint4 *>(a.O[0] + row_off + c) = make_uint4(w0[0], w0[1], w0[2], w0[3]);
+                *reinterpret_cast<uint4 *>(a.O[1] + row_off + c) = make_uint4(w1[0], w1[1], w1[2], w1[3]);
+                *reinterpret_cast<uint4 *>(a.O[2] + row_off + c) = make_uint4(w2[0], w2[1], w2[2], w2[3]);
             }
         }
     }
@@ -416,7 +443,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     __syncthreads();
     if (warp == 0 && lane == 0) {
         // nothing may still land in shared memory after exit
-        mbar_wait(smem_u32(&q_full), 0, a.err, SITE_AT_DRAIN);
         const int issued = s_issued;
         for (int j = issued - AT_STAGES < 0 ? 0 : issued - AT_STAGES; j < issued; ++j)
             mbar_wait(smem_u32(&kv_full[j % AT_STAGES]), (j / AT_STAGES) & 1, a.err, SITE_AT_DRAIN);

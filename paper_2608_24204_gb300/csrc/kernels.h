@@ -46,7 +46,6 @@ struct Bufs {
 // TMA descriptors of the prefill GEMM operands (built once per context).
 struct PrefillMaps {
     CUtensorMap a[kTerms], o[kTerms], m[kTerms];       // GEMM activations, 128-row boxes
-    CUtensorMap q[kTerms];                             // queries: [token][head][d], group x tpt boxes
     CUtensorMap kv;                                    // the whole KV pool: [page][K|V][kv_head][16][d]
     std::vector<CUtensorMap> wqkv, wo, wgu, wd;        // per layer weights, boxes of bn_* rows
     CUtensorMap wt_qkv[kTerms], wt_o[kTerms], wt_gu[kTerms], wt_d[kTerms];  // 8-bit format: the dequantised terms

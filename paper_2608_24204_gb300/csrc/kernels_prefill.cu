@@ -423,19 +423,6 @@ static bool encode_2d(CUtensorMap *m, const void *ptr, int rows, int K, int box_
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// queries [token][head][d] bf16: boxes of 64 d x `group` heads x tpt tokens (128-byte rows)
-static bool encode_q(CUtensorMap *m, const void *ptr, const Plan &p, int tpt) {
-    EncodeTiledFn enc = encode_fn();
-    if (!enc) return false;
-    cuuint64_t dims[3] = {(cuuint64_t)p.d, (cuuint64_t)p.nq, (cuuint64_t)p.max_chunk};
-    cuuint64_t strides[2] = {(cuuint64_t)p.d * 2, (cuuint64_t)p.qdim * 2};
-    cuuint32_t box[3] = {64, (cuuint32_t)p.group, (cuuint32_t)tpt};
-    cuuint32_t es[3] = {1, 1, 1};
-    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box, es,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 // the KV pool of every layer as [page (layer-major)][K|V][kv head][16 slots][d]:
 // boxes of 64 d x 16 slots of one (page, K|V, head)
 static bool encode_kv(CUtensorMap *m, const void *ptr, const Plan &p) {
@@ -455,10 +442,9 @@ static bool encode_kv(CUtensorMap *m, const void *ptr, const Plan &p) {
 const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
     const int T = p.max_chunk;
     bool ok = true;
-    const int tpt = attn_tokens_per_tile(p.group);
     for (int t = 0; t < kTerms; ++t)
         ok = ok && encode_2d(&m->a[t], b.A[t], T, p.H, TC_BM) && encode_2d(&m->o[t], b.O[t], T, p.qdim, TC_BM) &&
-             encode_2d(&m->m[t], b.M[t], T, p.F, TC_BM) && encode_q(&m->q[t], b.Q[t], p, tpt);
+             encode_2d(&m->m[t], b.M[t], T, p.F, TC_BM);
     if (!ok) return "cuTensorMapEncodeTiled failed for an activation operand";
     ok = encode_kv(&m->kv, b.KV, p);
     if (!ok) return "cuTensorMapEncodeTiled failed for the attention operands";
@@ -515,6 +501,7 @@ const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
 cudaError_t launch_attn_tc(const Plan &p, const Bufs &b, const PrefillMaps &mp, int layer, int P, int T,
                            cudaStream_t st) {
     AttnArgs a;
+    for (int t = 0; t < AT_TERMS; ++t) a.Q[t] = b.Q[t];
     for (int t = 0; t < kTerms; ++t) a.O[t] = b.O[t];
     a.pages = b.pages;
     a.err = b.ctrl + CTRL_ERR;
@@ -528,11 +515,9 @@ cudaError_t launch_attn_tc(const Plan &p, const Bufs &b, const PrefillMaps &mp, 
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)p.d);
     dim3 grid((T + a.tpt - 1) / a.tpt, p.nkv);
     if (p.d == 128)
-        attn_tc_kernel<128><<<grid, AT_THREADS, AttnSmem<128>::TOTAL + 1024, st>>>(mp.q[0], mp.q[1], mp.kv,
-                                                                                  a);
+        attn_tc_kernel<128><<<grid, AT_THREADS, AttnSmem<128>::TOTAL + 1024, st>>>(mp.kv, a);
     else
-        attn_tc_kernel<64><<<grid, AT_THREADS, AttnSmem<64>::TOTAL + 1024, st>>>(mp.q[0], mp.q[1], mp.kv,
-                                                                                a);
+        attn_tc_kernel<64><<<grid, AT_THREADS, AttnSmem<64>::TOTAL + 1024, st>>>(mp.kv, a);
     return cudaGetLastError();
 }
 
