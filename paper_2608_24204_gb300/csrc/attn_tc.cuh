@@ -3,31 +3,31 @@
 // One CTA computes causal GQA attention for a tile of query rows of one KV
 // head g: the rows pack TPT tokens x `group` query heads (row r = token r/group,
 // head g*group + r%group), so each K/V tile serves the whole group.  Keys come
-// from the paged cache in blocks of 64 (four 16-key pages, fetched by 5-D TMA
+// from the paged cache in blocks of 128 (eight 16-key pages, fetched by 5-D TMA
 // through the page table).  Per block j:
-//   S_j  = (Q_0 + Q_1) K_j^T      tcgen05.mma, M=128 rows, N=64 keys, fp32 in TMEM
+//   S_j  = (Q_0 + Q_1) K_j^T      tcgen05.mma, M=128 rows, N=128 keys, fp32 in TMEM
 //   softmax (one row per thread pair, read from TMEM): P_j = exp2(s - m), with m
-//          the row's reference maximum
+//          the row's reference maximum, stored over S_j in TMEM
 //   O   += (P_0 + P_1) V_j        tcgen05.mma, N=d, V read as an MN-major operand,
 //          accumulated in TMEM over all blocks
 // Both A operands live in tensor memory: the softmax warps store the tile's Q
-// terms there once, and each block's P terms next to S.  Shared memory then only
-// holds the K/V ring, and the tensor cores read only K and V from it (an N=64
-// MMA that also read its A operand from shared memory would need more than the
-// 128 bytes per clock that shared memory delivers).
+// terms there once, and each block's P terms over its S.  Shared memory only
+// holds the K/V ring, and the tensor cores read only K and V from it.  N=128
+// MMAs run at the full tensor rate (an N=64 one takes about 1.4 times its share).
 // The reference maximum only moves when a block's maximum exceeds it by more
 // than 2^8 (so P <= 256): then the softmax rescales its rows of the TMEM
 // accumulator and its row sums by exp2(m_old - m_new), between P_{j-1} V_{j-1}
 // and P_j V_j; the result O / l is the same softmax in exact arithmetic.
-// S and P are double-buffered, so the tensor cores work ahead of the softmax:
-// the MMA warp issues S_{j+2} as soon as the softmax has consumed S_j, and
-// P_j V_j runs while the softmax computes P_{j+1}.
+// S / P is double-buffered, so the tensor cores work ahead of the softmax: the
+// MMA warp issues S_{j+2} into buffer j % 2 right after P_j V_j (the tensor core
+// runs one thread's MMAs in issue order, so P_j is read before S_{j+2} lands),
+// and P_j V_j runs while the softmax computes P_{j+1}.
 // Q and P are carried as two bf16 terms (hi + lo: 16 significant bits), K and V
 // are exact bf16: the products only meet bf16 K and V, whose own rounding is 2^-9.
 // Warp roles: 0 TMA producer, 1 TMEM owner + MMA issuer, 2..9 softmax / output:
-// two warps per TMEM lane quadrant (warp % 4), one for keys 0..31, d values
+// two warps per TMEM lane quadrant (warp % 4), one for keys 0..63, d values
 // [0, d/2) of Q and output columns [0, d/2) of its 32 rows, the other for keys
-// 32..63 and the upper halves; the pair exchanges each block's row maxima
+// 64..127 and the upper halves; the pair exchanges each block's row maxima
 // through shared memory.  Every wait is bounded.
 #pragma once
 #include <cuda.h>
@@ -40,8 +40,8 @@
 namespace wici {
 
 constexpr int AT_ROWS = 128;           // query rows per tile (TMEM lanes)
-constexpr int AT_KEYS = 64;            // keys per block
-constexpr int AT_STAGES = 6;           // K/V ring depth
+constexpr int AT_KEYS = 128;           // keys per block
+constexpr int AT_STAGES = 3;           // K/V ring depth
 constexpr int AT_TERMS = 2;            // bf16 terms of the Q and P operands
 constexpr int AT_THREADS = 320;        // producer, MMA, 8 softmax warps (two per TMEM lane quadrant)
 constexpr uint32_t AT_TMEM_COLS = 512;
@@ -50,13 +50,14 @@ constexpr float AT_RESCALE_LOG2 = 8.f; // the reference maximum trails the row m
 enum : int { SITE_AT_Q = 41, SITE_AT_KVE = 42, SITE_AT_KVF = 43, SITE_AT_S = 44, SITE_AT_P = 45, SITE_AT_O = 46,
              SITE_AT_DRAIN = 47 };
 
-// TMEM columns (one 32-bit column holds two bf16 of a row): Q terms [0, d),
-// S buffers [d, d + 128), P buffers (two terms of 32 columns each) [d + 128, d + 256),
-// the O accumulator [d + 256, 2d + 256)
+// TMEM columns (one 32-bit column holds two bf16 of a row): Q terms [0, d);
+// S / P buffers [d, d + 128) and [d + 128, d + 256), each holding S (128 fp32
+// columns) and then P (term t in columns [64 t, 64 t + 64)); the O accumulator
+// [d + 256, 2d + 256)
 template <int D>
 struct AttnTmem {
-    static constexpr uint32_t Q = 0, S = D, P = D + 128, O = D + 256;
-    static_assert(2 * D + 256 <= (int)AT_TMEM_COLS, "tensor memory");
+    static constexpr uint32_t Q = 0, SP = D, O = D + 2 * AT_KEYS;
+    static_assert(2 * D + 2 * AT_KEYS <= (int)AT_TMEM_COLS, "tensor memory");
 };
 
 template <int D>
@@ -212,7 +213,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = s_tmem;
-    const uint32_t tm_q = tmem + TM::Q, tm_s = tmem + TM::S, tm_p = tmem + TM::P, tm_o = tmem + TM::O;
+    const uint32_t tm_q = tmem + TM::Q, tm_sp = tmem + TM::SP, tm_o = tmem + TM::O;
 
     if (warp == 0) {
         if (lane == 0) {  // ----------------------------------------------- TMA producer
@@ -231,7 +232,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                     const int pp = lp < a.max_pages ? a.pages[lp] : 0;   // past the table: masked keys
                     const int page = a.layer * a.max_pages + pp;
                     for (int c = 0; c < L::DCH; ++c) {
-                        // chunk c holds d values [64c, 64c+64) of all 64 keys (rows of 128 B)
+                        // chunk c holds d values [64c, 64c+64) of the block's keys (rows of 128 B)
                         tma_load_5d(kdst + c * (AT_KEYS * 128) + pg * 16 * 128, &map_kv, c * 64, 0, g, 0, page, fb);
                         tma_load_5d(vdst + c * (AT_KEYS * 128) + pg * 16 * 128, &map_kv, c * 64, 0, g, 1, page, fb);
                     }
@@ -251,7 +252,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                 if (!ok) return;
                 tc_fence_after();
                 const uint32_t kb = base + L::OFF_KV + (uint32_t)s * 2 * L::KV_BYTES;
-                const uint32_t sacc = tm_s + 64u * (uint32_t)(j & 1);
+                const uint32_t sacc = tm_sp + (uint32_t)AT_KEYS * (uint32_t)(j & 1);
 #pragma unroll
                 for (int k = 0; k < D / 16; ++k) {
                     // d values 16k..16k+15: 8 TMEM columns of each Q term, 32 bytes of each K row
@@ -267,21 +268,24 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             if (nb > 1) issue_s(1);
             for (int j = 0; j < nb && ok; ++j) {
                 const int s = j % AT_STAGES, b = j & 1;
-                // P_j stored (and S_j read, and O rescaled if its reference maximum moved) by the softmax
+                // P_j stored over S_j (and O rescaled if its reference maximum moved) by the softmax
                 ok = mbar_wait(smem_u32(&p_full[b]), (j >> 1) & 1, a.err, SITE_AT_P);
                 if (!ok) break;
                 tc_fence_after();
                 const uint32_t vb = base + L::OFF_KV + (uint32_t)s * 2 * L::KV_BYTES + L::KV_BYTES;
+                const uint32_t pb = tm_sp + (uint32_t)AT_KEYS * (uint32_t)b;
 #pragma unroll
                 for (int k = 0; k < AT_KEYS / 16; ++k) {
                     // 16 keys = two 8-key groups of V rows; P columns 8k..8k+7 of each term
                     const uint64_t vd = at_desc_mn(vb + 2048u * k, AT_KEYS * 128);
 #pragma unroll
                     for (int t = 0; t < AT_TERMS; ++t)
-                        tc_mma_ts(tm_o, tm_p + 64u * (uint32_t)b + 32u * t + 8u * k, vd, idesc_o, (j | k | t) != 0);
+                        tc_mma_ts(tm_o, pb + (uint32_t)(AT_KEYS / 2) * t + 8u * k, vd, idesc_o, (j | k | t) != 0);
                 }
-                tc_commit(smem_u32(&o_full));
                 tc_commit(smem_u32(&kv_empty[s]));
+                // the softmax waits for O only before its last block and at the end; earlier
+                // rescales wait for S_{j+1}, which lands after P_{j-1} V_{j-1}
+                if (j >= nb - 2) tc_commit(smem_u32(&o_full));
                 if (j + 2 < nb) issue_s(j + 2);   // S buffer b was read before P_j was posted
             }
         }
@@ -324,10 +328,12 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         bool ok = true;
         const uint32_t tm_orow = tm_o + lane_base + hc * HD;
         for (int j = 0; j < nb; ++j) {
+            const uint32_t sp = tm_sp + (uint32_t)AT_KEYS * (uint32_t)(j & 1) + lane_base;
             ok = ok && mbar_wait(smem_u32(&s_full[j & 1]), (j >> 1) & 1, a.err, SITE_AT_S);
             tc_fence_after();
             float sv[HK];
-            tc_ld32(tm_s + 64u * (uint32_t)(j & 1) + lane_base + hc * HK, sv);
+#pragma unroll
+            for (int c0 = 0; c0 < HK; c0 += 32) tc_ld32(sp + hc * HK + c0, sv + c0);
             if (j >= first_masked) {
 #pragma unroll
                 for (int c = 0; c < HK; ++c) {
@@ -342,7 +348,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             // the row's block maximum over both halves (raw scores: the scale is positive)
             s_rowmax[hc][r] = bm;
             // the pair leaves the loop together: the barrier also ANDs the two warps'
-            // wait results, so a wait that gave up in one warp never strands the other
+            // wait results, so a wait that gave up in one warp never strands the other.
+            // Past it both warps hold their S values in registers, so P may overwrite S.
             uint32_t both_ok;
             asm volatile(
                 "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 q, %1, 0;\n\t"
@@ -362,29 +369,36 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             const float mn = grow ? bm : m;
             const float corr = grow ? fast_exp2(m - mn) : 1.f;
             const float nms = mn == -INFINITY ? 0.f : -mn;   // rows with nothing visible yet
-            float ps = 0.f;
-            // P as two bf16 terms: this half's 32 keys are 16 columns of each term
-            uint32_t w0[HK / 2], w1[HK / 2];
+            float ps0 = 0.f, ps1 = 0.f;
+            // P as two bf16 terms over S: this half's 64 keys are 32 columns of each term,
+            // written 16 columns (32 keys) at a time
 #pragma unroll
-            for (int e = 0; e < HK / 2; ++e) {
-                const float p0 = fast_exp2(fmaf(sv[2 * e], a.scale_log2, nms));
-                const float p1 = fast_exp2(fmaf(sv[2 * e + 1], a.scale_log2, nms));
-                ps += p0 + p1;
-                w0[e] = pack_bf16x2(p0, p1);
-                w1[e] = pack_bf16x2(p0 - bf16lo(w0[e]), p1 - bf16hi(w0[e]));
+            for (int c0 = 0; c0 < HK; c0 += 32) {
+                uint32_t w0[16], w1[16];
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const float p0 = fast_exp2(fmaf(sv[c0 + 2 * e], a.scale_log2, nms));
+                    const float p1 = fast_exp2(fmaf(sv[c0 + 2 * e + 1], a.scale_log2, nms));
+                    ps0 += p0;
+                    ps1 += p1;
+                    w0[e] = pack_bf16x2(p0, p1);
+                    w1[e] = pack_bf16x2(p0 - bf16lo(w0[e]), p1 - bf16hi(w0[e]));
+                }
+                const uint32_t pc = sp + (uint32_t)(hc * (HK / 2) + c0 / 2);
+                tc_st16(pc, w0);
+                tc_st16(pc + AT_KEYS / 2, w1);
             }
-            // P buffer j & 1 is free: S_j completing means P_{j-2} V_{j-2} has too
-            const uint32_t prow = tm_p + 64u * (uint32_t)(j & 1) + lane_base + (uint32_t)hc * (HK / 2);
-            tc_st16(prow, w0);
-            tc_st16(prow + 32, w1);
             // O is rescaled once P_{j-1} V_{j-1} has landed and before P_j V_j is issued.
-            // Here o_full has completed j - 1 or j phases (S_j completing implies
-            // P_{j-2} V_{j-2} did; P_j is not posted), so its parity wait is exact even
-            // when earlier iterations skipped it; the last iteration always waits, which
-            // keeps the final wait below exact too.
+            // Before block nb - 1, S_{j+1} completing implies it (S_{j+1} was issued after
+            // it; P_{j+1} is not posted, so that parity wait is exact).  The last block
+            // always waits for the first of the two o_full phases (P_{nb-2} V_{nb-2}),
+            // which keeps the final wait for the second one exact.
             const bool any_grow = __any_sync(0xFFFFFFFFu, grow);
             if (j > 0 && (any_grow || j == nb - 1)) {
-                ok = ok && mbar_wait(smem_u32(&o_full), (j - 1) & 1, a.err, SITE_AT_O);
+                if (j + 1 < nb)
+                    ok = ok && mbar_wait(smem_u32(&s_full[(j + 1) & 1]), ((j + 1) >> 1) & 1, a.err, SITE_AT_O);
+                else
+                    ok = ok && mbar_wait(smem_u32(&o_full), 0, a.err, SITE_AT_O);
                 tc_fence_after();
                 if (any_grow) {
 #pragma unroll
@@ -399,7 +413,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                 }
             }
             tc_wait_st();
-            l = l * corr + ps;        // this half's share of the row sum, in the reference scale
+            l = l * corr + (ps0 + ps1);   // this half's share of the row sum, in the reference scale
             m = mn;
             tc_fence_before();
             __syncwarp();
@@ -410,7 +424,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
 #pragma unroll
         for (int i = 0; i < HD; ++i) o[i] = 0.f;
         if (ok && nb > 0) {
-            ok = mbar_wait(smem_u32(&o_full), (nb - 1) & 1, a.err, SITE_AT_O);
+            // o_full completes after P_{nb-2} V_{nb-2} (when nb > 1; waited for in the last
+            // block) and after P_{nb-1} V_{nb-1}
+            ok = mbar_wait(smem_u32(&o_full), nb > 1 ? 1 : 0, a.err, SITE_AT_O);
             tc_fence_after();
 #pragma unroll
             for (int c0 = 0; c0 < HD; c0 += 32) tc_ld32(tm_orow + c0, o + c0);
