@@ -53,12 +53,13 @@ constexpr size_t TC_SMEM_BUDGET = 216 * 1024;                           // ring 
 // geometry of a 128 x BN output tile whose stages hold AT activation terms
 template <int BN, int AT = kTerms>
 struct TcTile {
-    static_assert(BN % 64 == 0 && BN <= 256, "BN: a multiple of 64 up to 256");
+    static_assert(BN % 32 == 0 && BN <= 256, "BN: a multiple of 32 up to 256");
     static constexpr uint32_t B_BYTES = BN * TC_BK * 2;
     static constexpr uint32_t STAGE_BYTES = AT * TC_A_BYTES + B_BYTES;
     static constexpr int STAGES = (int)(TC_SMEM_BUDGET / STAGE_BYTES);
     static constexpr size_t SMEM = (size_t)STAGES * STAGE_BYTES + 1024;
     static constexpr int EPI_COLS = BN / 2;                               // columns per epilogue warp
+    static constexpr uint32_t ACC_STRIDE = TC_TMEM_COLS / 2;              // TMEM columns between the two buffers
     static_assert(STAGES >= 3, "at least three ring stages");
 };
 
@@ -109,6 +110,20 @@ __device__ __forceinline__ void tc_mma(uint32_t tmem_d, uint64_t adesc, uint64_t
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
                  : "memory");
+}
+
+// 16 consecutive fp32 columns of this thread's TMEM lane
+__device__ __forceinline__ void tc_ld16(uint32_t taddr, float *v) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
 // 32 consecutive fp32 columns of this thread's TMEM lane
@@ -214,7 +229,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     if (gg >= 2 && !(ok = mbar_wait(smem_u32(&acc_free[b]), ((gg / 2) + 1) & 1, err, SITE_TC_FREE)))
                         break;
                     tc_fence_after();
-                    const uint32_t acc = tmem + (uint32_t)(b * BN);
+                    const uint32_t acc = tmem + (uint32_t)b * G::ACC_STRIDE;
                     const int kk1 = min(nkk, (gi + 1) * TC_GROUP);
                     for (int kk = gi * TC_GROUP; kk < kk1; ++kk, ++it) {
                         const int s = it % S;
@@ -256,12 +271,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                 ok = mbar_wait(smem_u32(&acc_full[b]), (gg / 2) & 1, err, SITE_TC_ACCUM);
                 if (!ok) break;
                 tc_fence_after();
+                const uint32_t ta = tmem + lane_base + (uint32_t)b * G::ACC_STRIDE + (uint32_t)(half * G::EPI_COLS);
 #pragma unroll
-                for (int c0 = 0; c0 < G::EPI_COLS; c0 += 32) {
+                for (int c0 = 0; c0 + 32 <= G::EPI_COLS; c0 += 32) {
                     float v[32];
-                    tc_ld32(tmem + lane_base + (uint32_t)(b * BN + half * G::EPI_COLS + c0), v);
+                    tc_ld32(ta + (uint32_t)c0, v);
 #pragma unroll
                     for (int i = 0; i < 32; ++i) sum[c0 + i] += v[i];
+                }
+                if constexpr (G::EPI_COLS % 32 != 0) {   // a last 16 columns
+                    constexpr int c0 = G::EPI_COLS - 16;
+                    float v[16];
+                    tc_ld16(ta + (uint32_t)c0, v);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) sum[c0 + i] += v[i];
                 }
                 tc_fence_before();
                 __syncwarp();

@@ -19,12 +19,23 @@ namespace wici {
 // output-tile widths of the prefill GEMMs: 128 x 192 tiles (three 72 KB ring
 // stages) or 128 x 128 tiles (three 64 KB stages), chosen per weight matrix
 // for the fewest whole waves of tiles at the largest chunk
-static int pick_bn(int T, int N, int sms) {
+// output-tile width: the fewest columns per SM over the waves of tiles, a
+// 128-column tile charged 10% for reading its A operand more often per FLOP;
+// 224 only for GEMMs of two activation terms (three leave too few ring stages)
+static int pick_bn(int T, int N, int sms, bool allow224) {
     const int tm = (T + TC_BM - 1) / TC_BM;
-    const int w192 = (tm * ((N + 191) / 192) + sms - 1) / sms;
-    const int w128 = (tm * ((N + 127) / 128) + sms - 1) / sms;
-    // a narrower tile reads its A operand more often per FLOP: charge it 10%
-    return (double)w128 * 128 * 1.1 < (double)w192 * 192 ? 128 : 192;
+    int best = 0;
+    double best_cost = 0.0;
+    for (int bn : {128, 192, 224}) {
+        if (bn == 224 && !allow224) continue;
+        const int waves = (tm * ((N + bn - 1) / bn) + sms - 1) / sms;
+        const double cost = (double)waves * bn * (bn == 128 ? 1.1 : 1.0);
+        if (best == 0 || cost < best_cost) {
+            best = bn;
+            best_cost = cost;
+        }
+    }
+    return best;
 }
 
 // store a as its three bf16 terms
@@ -448,10 +459,10 @@ const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
     if (!ok) return "cuTensorMapEncodeTiled failed for an activation operand";
     ok = encode_kv(&m->kv, b.KV, p);
     if (!ok) return "cuTensorMapEncodeTiled failed for the attention operands";
-    m->bn_qkv = pick_bn(T, p.nqkv, p.num_sms);
-    m->bn_o = pick_bn(T, p.H, p.num_sms);
-    m->bn_gu = pick_bn(T, 2 * p.F, p.num_sms);
-    m->bn_d = pick_bn(T, p.H, p.num_sms);
+    m->bn_qkv = pick_bn(T, p.nqkv, p.num_sms, PEpiQKV::kATerms == 2);
+    m->bn_o = pick_bn(T, p.H, p.num_sms, PEpiResidual::kATerms == 2);
+    m->bn_gu = pick_bn(T, 2 * p.F, p.num_sms, PEpiSwiGLU::kATerms == 2);
+    m->bn_d = pick_bn(T, p.H, p.num_sms, PEpiResidual::kATerms == 2);
     if (p.q8) {
         // the 8-bit format: every GEMM reads the one dequantised matrix in the workspace
         for (int t = 0; t < kTerms; ++t) {
@@ -486,6 +497,8 @@ const char *make_prefill_maps(const Plan &p, const Bufs &b, PrefillMaps *m) {
             !WICI_GEMM_ATTR(192, kTerms, PEpiQKV) || !WICI_GEMM_ATTR(192, kTerms, PEpiResidual) ||
             !WICI_GEMM_ATTR(192, kTerms, PEpiSwiGLU) || !WICI_GEMM_ATTR(128, kTerms, PEpiQKV) ||
             !WICI_GEMM_ATTR(128, kTerms, PEpiResidual) || !WICI_GEMM_ATTR(128, kTerms, PEpiSwiGLU) ||
+            !WICI_GEMM_ATTR(224, 1, PEpiResidual) || !WICI_GEMM_ATTR(224, 1, PEpiSwiGLU) ||
+            !WICI_GEMM_ATTR(224, kTerms, PEpiResidual) || !WICI_GEMM_ATTR(224, kTerms, PEpiSwiGLU) ||
             cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)(AttnSmem<128>::TOTAL + 1024)) != cudaSuccess ||
             cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -546,8 +559,12 @@ static cudaError_t gemm(const Plan &p, int bn, const CUtensorMap *a, const WOper
     if (hook) hook->before(name);
     if (bn == 128)
         launch_gemm<128>(p, a, w, T, N, K, err, epi, st);
-    else
+    else if (bn == 192)
         launch_gemm<192>(p, a, w, T, N, K, err, epi, st);
+    else if constexpr (Epi::kATerms == 2)
+        launch_gemm<224>(p, a, w, T, N, K, err, epi, st);
+    else
+        return cudaErrorInvalidValue;   // pick_bn never picks 224 for three terms
     if (hook) hook->after(name);
     return cudaGetLastError();
 }
