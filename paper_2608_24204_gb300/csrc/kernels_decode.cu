@@ -1847,7 +1847,7 @@ using MegaF12288 = GShape<6, 1, true>;    // Qwen3-8B widths: hidden 4096, ffn 1
 // 8-bit block format: 16-element chunks per thread (NCH = ceil(K / 4096)), and
 // rows of q8_row_bytes(K) bytes per 32 KB slot: as many as fit, even where a
 // unit is a row pair
-using Q8H4096 = GShape<1, 6, true>;       // 6 x 4352 B
+using Q8H4096 = GShape<1, 7, true>;       // 7 x 4352 B
 using Q8F14336 = GShape<4, 2, false>;     // 2 x 15232 B; 896 chunks
 using Q8Small = GShape<1, 8, false>;      // 8 x <= 1904 B (K < 2048)
 using Q8F12288 = GShape<3, 2, true>;      // 2 x 13056 B
