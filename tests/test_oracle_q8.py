@@ -97,3 +97,22 @@ def test_tiny_model_in_the_8bit_format_matches_the_torch_restatement():
     assert tok == int(np.argmax(want))
     plain, _ = oracle.OracleModel(cfg, w, max_tokens=64).prefill(prompt)
     assert not np.allclose(got, plain)   # the 8-bit matrices are really used
+
+
+def test_block_matvec_at_the_8b_layer_widths():
+    # K = 4096 (Wo) and K = 14336 (Wd), the widths the decode GEMV phases stream:
+    # the block-wise product against the dense product of the dequantised rows
+    cfg = gen.LLAMA_8B
+    xr = np.random.default_rng(5)
+    for name in ("layers.0.wo", "layers.0.wd"):
+        codes, scales = gq.make_q8_tensor(cfg, name)
+        codes, scales = codes[:384], scales[:384]
+        x = xr.standard_normal(codes.shape[1])
+        got = Q.q8_matvec(codes, scales, x)
+        want = Q.q8_dequantize(codes, scales) @ x
+        np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-14 * float(np.abs(want).max()))
+        # one row by the scalar definition, block by block
+        d = Q.fp16_bits_to_f64(scales[7])
+        acc = sum(d[b] * float(np.dot(codes[7, 32 * b:32 * b + 32].astype(np.float64), x[32 * b:32 * b + 32]))
+                  for b in range(codes.shape[1] // 32))
+        assert abs(got[7] - acc) <= 1e-12 * (1 + abs(acc))
