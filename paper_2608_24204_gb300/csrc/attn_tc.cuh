@@ -181,8 +181,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     __shared__ float s_rowmax[2][AT_ROWS];      // [key half][row]: each block's row maxima, the row sums at the end
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = blockIdx.y;
-    const int tile = gridDim.x - 1 - blockIdx.x;     // heaviest (latest) tiles first
+    // CTAs in launch order take the tiles heaviest (latest) first across all KV
+    // heads, so the last wave holds the lightest tiles of every head
+    const int nkv = a.nq / a.group;
+    const int g = (int)blockIdx.x % nkv;
+    const int tile = (int)(gridDim.x / nkv) - 1 - (int)blockIdx.x / nkv;
     const int t0 = tile * a.tpt;
     const int t_end = min(a.T, t0 + a.tpt);
     const int nkeys = a.P + t_end;                    // keys the tile's last token sees

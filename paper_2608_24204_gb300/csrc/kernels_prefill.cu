@@ -526,7 +526,7 @@ cudaError_t launch_attn_tc(const Plan &p, const Bufs &b, const PrefillMaps &mp, 
     a.layer = layer;
     a.max_pages = p.max_pages;
     a.scale_log2 = 1.4426950408889634f / sqrtf((float)p.d);
-    dim3 grid((T + a.tpt - 1) / a.tpt, p.nkv);
+    dim3 grid(((T + a.tpt - 1) / a.tpt) * p.nkv);
     if (p.d == 128)
         attn_tc_kernel<128><<<grid, AT_THREADS, AttnSmem<128>::TOTAL + 1024, st>>>(mp.kv, a);
     else
