@@ -59,20 +59,47 @@ __global__ void embed_rows_kernel(const uint16_t *E, const int *tok, float *X, i
 }
 
 // A[t] = X[t] / sqrt(mean(X[t]^2) + eps) * g, stored as three bf16 terms
-__global__ void rmsnorm_rows_kernel(const float *X, const uint16_t *g, const Terms A, int H, float eps) {
+// One CTA per row t: RMSNorm of x_t with gain g, stored as the first `nterms`
+// bf16 terms of the next GEMM's operand (its kATerms).  H % 8 == 0: 8-element
+// chunks, one 16-byte store per term.
+__global__ void rmsnorm_rows_kernel(const float *X, const uint16_t *g, const Terms A, int H, float eps,
+                                    int nterms) {
     __shared__ float s_part[32];
     const int t = blockIdx.x;
-    const float *x = X + (size_t)t * H;
+    const float4 *x = reinterpret_cast<const float4 *>(X + (size_t)t * H);
+    const int nc = H >> 3;
     float ss = 0.f;
-    for (int i = threadIdx.x; i < H; i += blockDim.x) ss = fmaf(x[i], x[i], ss);
+    for (int c = threadIdx.x; c < nc; c += blockDim.x) {
+        const float4 u = x[2 * c], v = x[2 * c + 1];
+        ss = fmaf(u.x, u.x, ss); ss = fmaf(u.y, u.y, ss); ss = fmaf(u.z, u.z, ss); ss = fmaf(u.w, u.w, ss);
+        ss = fmaf(v.x, v.x, ss); ss = fmaf(v.y, v.y, ss); ss = fmaf(v.z, v.z, ss); ss = fmaf(v.w, v.w, ss);
+    }
     ss = warp_sum(ss);
     if ((threadIdx.x & 31) == 0) s_part[threadIdx.x >> 5] = ss;
     __syncthreads();
     float tot = 0.f;
     for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += s_part[w];
     const float rinv = 1.0f / sqrtf(tot / (float)H + eps);
-    for (int i = threadIdx.x; i < H; i += blockDim.x)
-        split_store(A.p, (size_t)t * H + i, x[i] * rinv * bf16_to_f32(g[i]));
+    for (int c = threadIdx.x; c < nc; c += blockDim.x) {
+        const float4 u = x[2 * c], v = x[2 * c + 1];
+        const uint4 gw = reinterpret_cast<const uint4 *>(g)[c];
+        const float y[8] = {u.x * rinv * bf16lo(gw.x), u.y * rinv * bf16hi(gw.x), u.z * rinv * bf16lo(gw.y),
+                            u.w * rinv * bf16hi(gw.y), v.x * rinv * bf16lo(gw.z), v.y * rinv * bf16hi(gw.z),
+                            v.z * rinv * bf16lo(gw.w), v.w * rinv * bf16hi(gw.w)};
+        uint32_t w[kTerms][4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            uint16_t a0[kTerms], a1[kTerms];
+            split_bf16x3(y[2 * e], a0[0], a0[1], a0[2]);
+            split_bf16x3(y[2 * e + 1], a1[0], a1[1], a1[2]);
+#pragma unroll
+            for (int q = 0; q < kTerms; ++q) w[q][e] = (uint32_t)a0[q] | ((uint32_t)a1[q] << 16);
+        }
+        const size_t o = (size_t)t * H + 8 * (size_t)c;
+#pragma unroll
+        for (int q = 0; q < kTerms; ++q)
+            if (q < nterms) *reinterpret_cast<uint4 *>(A.p[q] + o) = make_uint4(w[q][0], w[q][1], w[q][2], w[q][3]);
+    }
 }
 
 // --------------------------------------------------------------- epilogues ----
@@ -594,7 +621,7 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
         uint16_t *kvl = b.KV + (size_t)l * p.kv_layer_elems;
         // A3 + A4: RMSNorm, QKV (+bias), RoPE, paged KV append
         const Terms A = {{b.A[0], b.A[1], b.A[2]}};
-        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.attn_norm, A, p.H, p.cfg.rms_eps);
+        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.attn_norm, A, p.H, p.cfg.rms_eps, PEpiQKV::kATerms);
         PEpiQKV eq = {{{b.Q[0], b.Q[1], b.Q[2]}}, kvl, b.pages, b.rope, p.cfg.qkv_bias ? b.W + lo.bqkv : nullptr, P, p.qdim,
                       p.kvdim, p.d, p.nkv, p.kv_page_elems, p.qk_norm ? b.QKraw : nullptr};
         WOperand w;
@@ -630,7 +657,7 @@ cudaError_t enqueue_prefill_chunk(const Plan &p, const Bufs &b, const PrefillMap
                       "prefill_o_proj")) != cudaSuccess)
             return e;
         // A7: RMSNorm + gate/up + SwiGLU
-        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.ffn_norm, A, p.H, p.cfg.rms_eps);
+        rmsnorm_rows_kernel<<<T, 256, 0, st>>>(b.X, b.W + lo.ffn_norm, A, p.H, p.cfg.rms_eps, PEpiSwiGLU::kATerms);
         const Terms M = {{b.M[0], b.M[1], b.M[2]}};
         if ((e = weight_operand<PEpiSwiGLU>(p, b, p.q8 ? mp.wt_gu[0] : mp.wgu[l], mp.wt_gu, b.W + lo.wgu, 2 * p.F, p.H, st,
                                 hook, &w)) != cudaSuccess)
