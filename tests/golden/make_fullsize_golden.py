@@ -7,7 +7,9 @@ hundreds of full-depth steps on the fly.  This script runs them once:
 
   * llama3-8b: the 1024-token prompt (seed 1), then 64 decode steps;
   * llama3-8b-agentic: 4 turns, each a 2048-token chunk (seeds 1..4) appended
-    to the same cache and then 64 decode steps, ending at 8448 cached tokens.
+    to the same cache and then 64 decode steps, ending at 8448 cached tokens;
+  * llama3.2-1b: the 512-token prompt (seed 1), then all 128 decode steps of
+    the configuration.
 
 Decode steps are teacher-forced with a seeded token sequence (seed 101 + turn,
 drawn like a prompt), so the oracle can take each turn's 64 steps as one causal
@@ -42,6 +44,7 @@ WORKLOADS = {
     # name: (config, decode steps per turn)
     "llama3-8b": (gen.LLAMA_8B, 64),
     "llama3-8b-agentic": (gen.LLAMA_8B_AGENTIC, 64),
+    "llama3.2-1b": (gen.LLAMA_1B, 128),
 }
 
 

@@ -2,8 +2,9 @@
 lengths, in the launch configuration the benchmark times (one prefill per
 chunk, then captured-graph decode steps), against the fp64 oracle.
 
-The Llama-3-8B request and the agentic workload are compared with oracle
-records stored under tests/golden/ (written by make_fullsize_golden.py, which
+The Llama-3-8B request, the agentic workload and the Llama-3.2-1B request
+(all 128 of its decode steps) are compared with oracle records stored under
+tests/golden/ (written by make_fullsize_golden.py, which
 runs only the oracle): every decode step is teacher-forced with the record's
 seeded tokens through `token_in`, and every produced logits vector is compared,
 in full at the recorded positions and at 1024 fixed sample indices plus the
@@ -28,13 +29,15 @@ if not torch.cuda.is_available():
 from paper_2608_24204_gb300 import WiciModel  # noqa: E402
 
 GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
-_w8b = {}
+_weights = {}
 
 
-def _weights_8b():
-    if "w" not in _w8b:
-        _w8b["w"] = gen.make_weights(gen.LLAMA_8B)
-    return _w8b["w"]
+def _weights_of(cfg):
+    key = tuple(gen.tensor_specs(cfg))          # configs of one shape share their weights
+    if key not in _weights:
+        _weights.clear()
+        _weights[key] = gen.make_weights(cfg)
+    return _weights[key]
 
 
 def _check_sampled(got, got_tok, rec, t, p, where, stats):
@@ -63,7 +66,7 @@ def _replay(name, max_tokens, max_chunk):
     cfg = gen.CONFIGS[str(rec["config"])]
     turns, steps, plen = int(rec["turns"]), int(rec["steps"]), int(rec["prompt_len"])
     full = {(int(t), int(p)): i for i, (t, p) in enumerate(rec["full_where"])}
-    model = WiciModel(cfg, max_tokens=max_tokens, max_chunk=max_chunk).load(_weights_8b())
+    model = WiciModel(cfg, max_tokens=max_tokens, max_chunk=max_chunk).load(_weights_of(cfg))
     stats, full_stats = {}, {}
 
     def compare(got, gtok, t, p, where):
@@ -98,7 +101,14 @@ def test_agentic_full_depth_four_turns_against_stored_oracle():
     # 32 layers, 4 x (2048-token chunk + 64 decode steps), 8448 cached at the end
     stats = _replay("llama3-8b-agentic", max_tokens=8448, max_chunk=2048)
     assert len(stats["max_abs"]) == 4 * 65
-    _w8b.clear()
+    _weights.clear()
+
+
+def test_llama32_1b_request_128_decode_steps_against_stored_oracle():
+    # the 1B configuration's whole request: 512-token prompt, then 128 decode steps
+    stats = _replay("llama3.2-1b", max_tokens=512 + 128 + 16, max_chunk=512)
+    assert len(stats["max_abs"]) == 129
+    _weights.clear()
 
 
 def _full(cfg, decode_steps, max_chunk=None):
