@@ -10,7 +10,7 @@ import threading
 
 import numpy as np
 
-from .configs import (CONFIGS, LLAMA_1B, LLAMA_8B, LLAMA_8B_AGENTIC, QWEN3_8B, QWEN_14B, TINY,
+from .configs import (CONFIGS, FALCON_40B, FALCON_TINY, LLAMA_1B, LLAMA_8B, LLAMA_8B_AGENTIC, QWEN3_8B, QWEN_14B, TINY,
                       ModelConfig, decode_bytes_per_token, prefill_flops, tensor_specs)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -101,6 +101,6 @@ def make_prompt(cfg: ModelConfig, n: int, seed: int = 1) -> np.ndarray:
     return out
 
 
-__all__ = ["CONFIGS", "TINY", "LLAMA_1B", "LLAMA_8B", "LLAMA_8B_AGENTIC", "QWEN_14B", "QWEN3_8B",
+__all__ = ["CONFIGS", "TINY", "LLAMA_1B", "LLAMA_8B", "LLAMA_8B_AGENTIC", "QWEN_14B", "QWEN3_8B", "FALCON_TINY", "FALCON_40B",
            "ModelConfig", "tensor_specs", "decode_bytes_per_token", "prefill_flops",
            "make_tensor", "make_weights", "make_prompt", "normal_f64", "draw", "stream", "build"]

@@ -26,6 +26,9 @@ class ModelConfig:
     tied_embeddings: bool = False
     qkv_bias: bool = False
     qk_norm: bool = False          # Qwen3 block: per-head RMSNorm of q and k before RoPE
+    # "llama": sequential attention then SwiGLU MLP, RMSNorm; "falcon": Falcon-40B's
+    # parallel attention and GELU MLP, each after its own LayerNorm (weight and bias)
+    block: str = "llama"
     weight_std: float = 0.02
     weight_seed: int = 0
     # workload: `turns` rounds of (prompt_len-token chunk, then decode_steps greedy tokens)
@@ -84,17 +87,34 @@ QWEN3_8B = ModelConfig(
     ffn_dim=12288, vocab=151936, rope_theta=1000000.0, rms_eps=1e-6, qk_norm=True,
     prompt_len=1024, decode_steps=256)
 
-CONFIGS = {c.name: c for c in (TINY, LLAMA_1B, LLAMA_8B, LLAMA_8B_AGENTIC, QWEN_14B, QWEN3_8B)}
+# The paper's largest evaluated model (Falcon-40B, Tab. 1): the Falcon block of
+# the public model family (parallel attention and MLP from one residual stream,
+# two LayerNorms per layer, a 4H GELU MLP, 128 query / 8 KV heads of 64,
+# rotate-half RoPE, tied embeddings), and a two-layer stand-in for the pins.
+FALCON_40B = ModelConfig(
+    name="falcon-40b", n_layers=60, hidden=8192, n_q_heads=128, n_kv_heads=8, head_dim=64,
+    ffn_dim=32768, vocab=65024, rope_theta=10000.0, rms_eps=1e-5, tied_embeddings=True,
+    block="falcon", prompt_len=1024, decode_steps=256)
+
+FALCON_TINY = FALCON_40B.with_(
+    name="falcon-tiny", n_layers=2, hidden=256, n_q_heads=8, n_kv_heads=2, head_dim=32,
+    ffn_dim=1024, vocab=1024, prompt_len=32, decode_steps=16)
+
+CONFIGS = {c.name: c for c in (TINY, LLAMA_1B, LLAMA_8B, LLAMA_8B_AGENTIC, QWEN_14B, QWEN3_8B, FALCON_TINY,
+                               FALCON_40B)}
 
 
 def tensor_specs(cfg: ModelConfig):
     """Canonical tensor list: (name, (rows, cols), kind) with kind 'normal', 'ones'
-    or 'gain' (1 + 0.25 N(0, 1): the per-head q/k norm gains, not all one).
+    or 'gain' (1 + 0.25 N(0, 1): the per-head q/k norm gains and the Falcon
+    LayerNorm weights, not all one).
 
     The position of a tensor in this list is its generator tag.  All matrices
     are row-major [out, in]; y = W x.
     """
     H, d = cfg.hidden, cfg.head_dim
+    if cfg.block == "falcon":
+        return _falcon_specs(cfg)
     specs = [("embed", (cfg.vocab, H), "normal")]
     for l in range(cfg.n_layers):
         p = f"layers.{l}."
@@ -120,7 +140,32 @@ def tensor_specs(cfg: ModelConfig):
     return specs
 
 
-Q8_LAYER_MATRICES = ("wq", "wk", "wv", "wo", "wg", "wu", "wd")
+def _falcon_specs(cfg: ModelConfig):
+    """Falcon block: per layer a LayerNorm (weight ln_attn, bias ln_attn_b) for the
+    attention branch and one (ln_mlp, ln_mlp_b) for the MLP branch, no biases in
+    the matrices; MLP w_up [F, H], w_down [H, F]; a final LayerNorm."""
+    H, d = cfg.hidden, cfg.head_dim
+    specs = [("embed", (cfg.vocab, H), "normal")]
+    for l in range(cfg.n_layers):
+        p = f"layers.{l}."
+        specs.append((p + "ln_attn", (1, H), "gain"))
+        specs.append((p + "ln_attn_b", (1, H), "normal"))
+        specs.append((p + "ln_mlp", (1, H), "gain"))
+        specs.append((p + "ln_mlp_b", (1, H), "normal"))
+        specs.append((p + "wq", (cfg.n_q_heads * d, H), "normal"))
+        specs.append((p + "wk", (cfg.n_kv_heads * d, H), "normal"))
+        specs.append((p + "wv", (cfg.n_kv_heads * d, H), "normal"))
+        specs.append((p + "wo", (H, cfg.n_q_heads * d), "normal"))
+        specs.append((p + "w_up", (cfg.ffn_dim, H), "normal"))
+        specs.append((p + "w_down", (H, cfg.ffn_dim), "normal"))
+    specs.append(("final_norm", (1, H), "gain"))
+    specs.append(("final_norm_b", (1, H), "normal"))
+    if not cfg.tied_embeddings:
+        specs.append(("lm_head", (cfg.vocab, H), "normal"))
+    return specs
+
+
+Q8_LAYER_MATRICES = ("wq", "wk", "wv", "wo", "wg", "wu", "wd", "w_up", "w_down")
 
 
 def decode_bytes_per_token(cfg: ModelConfig, ctx: int, q8: bool = False) -> int:
@@ -147,7 +192,8 @@ def prefill_flops(cfg: ModelConfig, T: int, P: int = 0) -> float:
     2*T*(per-layer linear params)*L + causal attention (unmasked pairs only,
     QK^T and PV) + the LM head on the last row."""
     H, d = cfg.hidden, cfg.head_dim
-    lin = H * (cfg.q_dim + 2 * cfg.kv_dim) + cfg.q_dim * H + 3 * H * cfg.ffn_dim
+    mlp = (2 if cfg.block == "falcon" else 3) * H * cfg.ffn_dim     # GELU: up, down; SwiGLU: gate, up, down
+    lin = H * (cfg.q_dim + 2 * cfg.kv_dim) + cfg.q_dim * H + mlp
     pairs = T * P + T * (T + 1) // 2
     attn = cfg.n_q_heads * d * 4 * pairs
     return float(2 * T * lin * cfg.n_layers + attn * cfg.n_layers + 2 * cfg.vocab * H)

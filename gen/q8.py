@@ -22,7 +22,7 @@ from .configs import ModelConfig, tensor_specs
 Q8_BLOCK = 32
 Q8_CODE_TAG = 0x100000    # + the tensor's canonical tag: the codes' stream
 Q8_SCALE_TAG = 0x200000   # + the tensor's canonical tag: the scales' stream
-Q8_MATRICES = ("wq", "wk", "wv", "wo", "wg", "wu", "wd")   # per-layer matrices stored in the format
+Q8_MATRICES = ("wq", "wk", "wv", "wo", "wg", "wu", "wd", "w_up", "w_down")   # per-layer matrices in the format
 
 
 def q8_names(cfg: ModelConfig) -> list:

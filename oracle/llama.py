@@ -28,6 +28,13 @@ and listed with the same wording in the design notes:
   * Qwen3 block (`qk_norm`): each head of q and of k is RMS-normalised over
     head_dim with its own gain (q_norm, k_norm), after the projection and
     before RoPE.
+  * Falcon block (`block == "falcon"`, the Falcon-40B model of Tab. 1; the
+    block comes from the public model family, not from the paper): attention
+    and MLP both read the same residual stream x, each through its own
+    LayerNorm with weight and bias (ln_attn, ln_mlp), and both add to it:
+    x + Wo attn(LN_attn(x)) + W_down gelu(W_up LN_mlp(x)); GELU with the
+    exact erf; no biases in the matrices; a final LayerNorm with bias.
+    LayerNorm uses the biased variance over the hidden axis.
   * Greedy token = argmax of the logits, lowest index on an exact tie.
   * Optional `q8_weights`: matrices in the 8-bit block format (oracle/q8.py)
     replace the bf16 tensors of the same name.
@@ -93,6 +100,19 @@ def apply_rope(x: np.ndarray, cos: np.ndarray, sin: np.ndarray) -> np.ndarray:
 def silu(z: np.ndarray) -> np.ndarray:
     """silu(z) = z / (1 + exp(-z))."""
     return z / (1.0 + np.exp(-z))
+
+
+def layernorm(x: np.ndarray, g: np.ndarray, b: np.ndarray, eps: float) -> np.ndarray:
+    """(x - mean(x)) / sqrt(mean((x - mean(x))^2) + eps) * g + b over the last axis."""
+    c = x - np.mean(x, axis=-1, keepdims=True)
+    var = np.mean(c * c, axis=-1, keepdims=True)
+    return c / np.sqrt(var + eps) * g + b
+
+
+def gelu(z: np.ndarray) -> np.ndarray:
+    """gelu(z) = z * Phi(z) = z / 2 * (1 + erf(z / sqrt(2))), with the exact erf."""
+    from scipy.special import erf
+    return 0.5 * z * (1.0 + erf(z / np.sqrt(2.0)))
 
 
 def softmax(s: np.ndarray, axis: int = -1) -> np.ndarray:
@@ -193,8 +213,12 @@ class OracleModel:
         cos, sin = rope_cos_sin(pos, d, cfg.rope_theta)
 
         x = bf16_bits_to_f64(self.w["embed"][tokens])                  # [T, H]
+        falcon = getattr(cfg, "block", "llama") == "falcon"
         for l in range(cfg.n_layers):
             p = f"layers.{l}."
+            if falcon:
+                x = self._falcon_layer(l, x, T, P, pos, cos, sin, rnd)
+                continue
             h = rnd(rmsnorm(x, self._vec(p + "attn_norm"), cfg.rms_eps))
             q = h @ self.W(p + "wq").T
             k = h @ self.W(p + "wk").T
@@ -222,10 +246,32 @@ class OracleModel:
             x = x + rnd(m) @ self.W(p + "wd").T
         self.kv_len = P + T
         lm = "embed" if cfg.tied_embeddings else "lm_head"
+        if falcon:
+            final = lambda a: layernorm(a, self._vec("final_norm"), self._vec("final_norm_b"), cfg.rms_eps)  # noqa: E731
+        else:
+            final = lambda a: rmsnorm(a, self._vec("final_norm"), cfg.rms_eps)  # noqa: E731
         if all_rows:
-            return rmsnorm(x, self._vec("final_norm"), cfg.rms_eps) @ self.W(lm).T
-        hf = rmsnorm(x[-1], self._vec("final_norm"), cfg.rms_eps)
-        return self.W(lm) @ hf
+            return final(x) @ self.W(lm).T
+        return self.W(lm) @ final(x[-1])
+
+    def _falcon_layer(self, l, x, T, P, pos, cos, sin, rnd):
+        """One Falcon block: x + Wo attn(LN_attn(x)) + W_down gelu(W_up LN_mlp(x))."""
+        cfg = self.cfg
+        d, n_q, n_kv = cfg.head_dim, cfg.n_q_heads, cfg.n_kv_heads
+        p = f"layers.{l}."
+        ha = rnd(layernorm(x, self._vec(p + "ln_attn"), self._vec(p + "ln_attn_b"), cfg.rms_eps))
+        hm = rnd(layernorm(x, self._vec(p + "ln_mlp"), self._vec(p + "ln_mlp_b"), cfg.rms_eps))
+        q = apply_rope((ha @ self.W(p + "wq").T).reshape(T, n_q, d), cos, sin)
+        k = apply_rope((ha @ self.W(p + "wk").T).reshape(T, n_kv, d), cos, sin)
+        v = (ha @ self.W(p + "wv").T).reshape(T, n_kv, d)
+        self.K[l][:, P:P + T, :] = round_bf16(k).transpose(1, 0, 2)
+        self.V[l][:, P:P + T, :] = round_bf16(v).transpose(1, 0, 2)
+        Kc = self.K[l][:, :P + T, :].astype(np.float64)
+        Vc = self.V[l][:, :P + T, :].astype(np.float64)
+        o = causal_gqa_attention(rnd(q), Kc, Vc, pos)
+        attn = rnd(o.reshape(T, n_q * d)) @ self.W(p + "wo").T
+        mlp = rnd(gelu(hm @ self.W(p + "w_up").T)) @ self.W(p + "w_down").T
+        return x + attn + mlp
 
     def prefill(self, tokens):
         logits = self.forward(tokens, round_act=self.prefill_act_bf16)

@@ -117,7 +117,10 @@ def _check(rc, ctx=None):
 
 def make_config(cfg, max_tokens: int, max_chunk: int | None = None, q8: bool = False,
                 max_sms: int = 0) -> wici_config:
-    """wici_config from a gen.ModelConfig-like object."""
+    """wici_config from a gen.ModelConfig-like object (Llama / Qwen blocks; the
+    library has no kernels for another block, such as Falcon's)."""
+    if getattr(cfg, "block", "llama") != "llama":
+        raise ValueError(f"{cfg.name}: the {cfg.block} block has no CUDA path in this library")
     return wici_config(cfg.n_layers, cfg.hidden, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.ffn_dim,
                        cfg.vocab, max_tokens, min(max_chunk or cfg.max_chunk, max_tokens), 16, cfg.rms_eps,
                        cfg.rope_theta, int(cfg.tied_embeddings), int(cfg.qkv_bias),
