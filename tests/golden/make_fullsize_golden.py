@@ -6,6 +6,7 @@ numpy in fp64 (tens of seconds on a CPU), so the GPU tests cannot recompute
 hundreds of full-depth steps on the fly.  This script runs them once:
 
   * llama3-8b: the 1024-token prompt (seed 1), then 64 decode steps;
+  * llama3-8b-256: the same prompt, then all 256 decode steps of the request;
   * llama3-8b-agentic: 4 turns, each a 2048-token chunk (seeds 1..4) appended
     to the same cache and then 64 decode steps, ending at 8448 cached tokens;
   * llama3.2-1b: the 512-token prompt (seed 1), then all 128 decode steps of
@@ -43,6 +44,7 @@ FORCED_SEED0 = 101
 WORKLOADS = {
     # name: (config, decode steps per turn)
     "llama3-8b": (gen.LLAMA_8B, 64),
+    "llama3-8b-256": (gen.LLAMA_8B, 256),
     "llama3-8b-agentic": (gen.LLAMA_8B_AGENTIC, 64),
     "llama3.2-1b": (gen.LLAMA_1B, 128),
 }

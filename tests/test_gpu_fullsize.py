@@ -2,9 +2,9 @@
 lengths, in the launch configuration the benchmark times (one prefill per
 chunk, then captured-graph decode steps), against the fp64 oracle.
 
-The Llama-3-8B request, the agentic workload and the Llama-3.2-1B request
-(all 128 of its decode steps) are compared with oracle records stored under
-tests/golden/ (written by make_fullsize_golden.py, which
+The Llama-3-8B request (64 and all 256 decode steps), the agentic workload
+and the Llama-3.2-1B request (all 128 of its decode steps) are compared with
+oracle records stored under tests/golden/ (written by make_fullsize_golden.py, which
 runs only the oracle): every decode step is teacher-forced with the record's
 seeded tokens through `token_in`, and every produced logits vector is compared,
 in full at the recorded positions and at 1024 fixed sample indices plus the
@@ -95,6 +95,12 @@ def test_llama3_8b_request_64_decode_steps_against_stored_oracle():
     # the bench's launch configuration: 1024-token prompt in one chunk, room for 256 steps
     stats = _replay("llama3-8b", max_tokens=1024 + 256 + 16, max_chunk=1024)
     assert len(stats["max_abs"]) == 65
+
+
+def test_llama3_8b_request_all_256_decode_steps_against_stored_oracle():
+    # the bench's whole request: 1024-token prompt, then all 256 decode steps
+    stats = _replay("llama3-8b-256", max_tokens=1024 + 256 + 16, max_chunk=1024)
+    assert len(stats["max_abs"]) == 257
 
 
 def test_agentic_full_depth_four_turns_against_stored_oracle():

@@ -11,7 +11,8 @@ import pytest
 import gen
 
 GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
-RECORDS = {"llama3-8b": (1, 1024, 64), "llama3-8b-agentic": (4, 2048, 64), "llama3.2-1b": (1, 512, 128)}
+RECORDS = {"llama3-8b": (1, 1024, 64), "llama3-8b-agentic": (4, 2048, 64), "llama3.2-1b": (1, 512, 128),
+           "llama3-8b-256": (1, 1024, 256)}
 
 
 @pytest.mark.parametrize("name", sorted(RECORDS))
