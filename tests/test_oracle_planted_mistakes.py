@@ -3,9 +3,11 @@ plants one (a flipped RoPE sign, a dropped norm gain, a wrong KV-head mapping,
 an off-by-one causal mask, a wrong softmax scale, the wrong RoPE frequency
 ladder, a missing bf16 rounding of the cache, norm gains swapped between the
 two branches, a missing Qwen3 q/k norm or Falcon LayerNorm mean, a sequential
-instead of parallel Falcon block) into a patched copy of oracle/llama.py on the
-CPU and checks that the independent torch restatements of the pins then
-disagree with it; the unpatched oracle agrees with them (the pins themselves).
+instead of parallel Falcon block; a shifted padding, stride or flipped taps in
+the convolution; unsigned codes or per-row scales in the 8-bit format) into a
+patched copy of the oracle on the CPU and checks that the independent torch restatements of the pins then
+(or the brute-force and library pins) then disagree with it; the unpatched
+oracle agrees with them (the pins themselves).
 The synthetic hidden-vector norm gains are all one, so the Llama cases run
 with non-unit gains.  Nothing here touches the CUDA path."""
 import numpy as np
@@ -156,3 +158,70 @@ def test_falcon_mistakes_are_caught(monkeypatch):
     with monkeypatch.context() as mp:
         mp.setattr(L.OracleModel, "_falcon_layer", sequential)
         assert np.abs(_oracle_logits(cfg, w, prompt) - want).max() > 100 * ATOL
+
+
+# ------------------------------------------------- convolution and 8-bit format
+def _conv_pin_error():
+    """max deviation of the conv oracle from F.conv2d and autograd (the pin)"""
+    import torch
+    import torch.nn.functional as F
+    from oracle import conv as C
+    r = np.random.default_rng(4)
+    x = torch.from_numpy(r.standard_normal((2, 10, 12, 5))).requires_grad_(True)
+    w = torch.from_numpy(r.standard_normal((4, 3, 3, 5))).requires_grad_(True)
+    dy = torch.from_numpy(r.standard_normal((2, 5, 6, 4)))
+    y = F.conv2d(x.permute(0, 3, 1, 2), w.permute(0, 3, 1, 2), stride=2, padding=1).permute(0, 2, 3, 1)
+    y.backward(dy)
+    xn, wn = x.detach().numpy(), w.detach().numpy()
+    return max(np.abs(C.conv_forward(xn, wn) - y.detach().numpy()).max(),
+               np.abs(C.conv_backward_data(dy.numpy(), wn, 10, 12) - x.grad.numpy()).max(),
+               np.abs(C.conv_backward_filter(xn, dy.numpy()) - w.grad.numpy()).max())
+
+
+def test_conv_mistakes_are_caught(monkeypatch):
+    from oracle import conv as C
+    assert _conv_pin_error() < 1e-10
+    with monkeypatch.context() as mp:     # padding on the far side only: every tap one pixel off
+        mp.setattr(C, "_padded", lambda x: np.pad(np.asarray(x, np.float64), ((0, 0), (0, 2), (0, 2), (0, 0))))
+        assert _conv_pin_error() > 1e-3
+    with monkeypatch.context() as mp:     # stride 1 sampling
+        mp.setattr(C, "STRIDE", 1)
+        assert _conv_pin_error() > 1e-3
+    real_fwd = C.conv_forward
+    with monkeypatch.context() as mp:     # taps flipped (a true convolution, not the correlation)
+        mp.setattr(C, "conv_forward", lambda x, w: real_fwd(x, np.asarray(w)[:, ::-1, ::-1, :]))
+        assert _conv_pin_error() > 1e-3
+
+
+def test_q8_mistakes_are_caught(monkeypatch):
+    import struct
+    from oracle import q8 as Q
+    r = np.random.default_rng(6)
+    codes = r.integers(-127, 128, size=(3, 96)).astype(np.int8)
+    scales = (r.uniform(0.5, 1.5, size=(3, 3)) * 1e-3).astype(np.float16).view(np.uint16)
+    x = r.standard_normal(96)
+
+    def pin_error():
+        # the brute-force pin: the block definition with an independent fp16 decoding
+        got = Q.q8_matvec(codes, scales, x)
+        want = [sum(struct.unpack("<e", struct.pack("<H", int(scales[i, b])))[0]
+                    * sum(int(codes[i, 32 * b + k]) * float(x[32 * b + k]) for k in range(32)) for b in range(3))
+                for i in range(3)]
+        return float(np.abs(got - np.array(want)).max())
+    assert pin_error() < 1e-12
+    with monkeypatch.context() as mp:     # codes read as unsigned bytes
+        mp.setattr(Q, "q8_matvec", _unsigned_matvec)
+        assert pin_error() > 1e-6
+    with monkeypatch.context() as mp:     # one scale per row instead of per block
+        mp.setattr(Q, "fp16_bits_to_f64", lambda b: np.repeat(np.asarray(b, np.uint16).view(np.float16)
+                                                              .astype(np.float64)[..., :1], np.asarray(b).shape[-1], -1))
+        assert pin_error() > 1e-6
+
+
+def _unsigned_matvec(codes, scales, x):
+    """the block product with the codes read as unsigned bytes (the planted mistake)"""
+    rows, cols = codes.shape
+    nb = cols // 32
+    q = np.asarray(codes).view(np.uint8).astype(np.float64).reshape(rows, nb, 32)
+    d = np.asarray(scales, np.uint16).view(np.float16).astype(np.float64).reshape(rows, nb)
+    return (np.einsum("rbk,bk->rb", q, np.asarray(x).reshape(nb, 32)) * d).sum(axis=1)
