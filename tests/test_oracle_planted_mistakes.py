@@ -1,15 +1,16 @@
 """The oracle's pins must catch a plausible mistake anywhere in it.  Each case
-plants one (a flipped RoPE sign, a dropped norm gain, a wrong KV-head mapping,
-an off-by-one causal mask, a wrong softmax scale, the wrong RoPE frequency
-ladder, a missing bf16 rounding of the cache, norm gains swapped between the
-two branches, a missing Qwen3 q/k norm or Falcon LayerNorm mean, a sequential
-instead of parallel Falcon block; a shifted padding, stride or flipped taps in
-the convolution; unsigned codes or per-row scales in the 8-bit format) into a
-patched copy of the oracle on the CPU and checks that the independent torch restatements of the pins then
-(or the brute-force and library pins) then disagree with it; the unpatched
-oracle agrees with them (the pins themselves).
-The synthetic hidden-vector norm gains are all one, so the Llama cases run
-with non-unit gains.  Nothing here touches the CUDA path."""
+plants one into a patched copy of the oracle on the CPU and checks that the
+pins (the independent torch restatements, the brute-force and library
+comparisons) then disagree with it, while the unpatched oracle agrees with
+them.  The mistakes: a flipped RoPE sign, the wrong RoPE frequency ladder, a
+dropped norm gain, norm gains swapped between the two branches, a wrong
+KV-head mapping, an off-by-one causal mask, a wrong softmax scale, a missing
+bf16 rounding of the cache, silu as the identity, a missing Qwen3 q/k norm, a
+LayerNorm without its mean, a tanh GELU, a sequential Falcon block; a shifted
+padding, stride 1 or flipped taps in the convolution; unsigned codes or
+per-row scales in the 8-bit format.  The synthetic hidden-vector norm gains
+are all one, so the Llama cases run with non-unit gains.  Nothing here touches
+the CUDA path."""
 import numpy as np
 import pytest
 
